@@ -1,0 +1,146 @@
+"""Plant plausible mistakes in the oracle (on the CPU) and check that the
+pins of test_oracle_pins catch every one of them: the pins are only worth
+something if a dropped term, a wrong sign, a swapped index or an off-by-one
+in the oracle makes at least one of them fail."""
+import math
+
+import numpy as np
+import pytest
+
+from oracle import mmshift_oracle as O
+from tests import test_oracle_pins as P
+
+
+def _window_stats_ddof0(qwin):
+    q = np.asarray(qwin, dtype=np.float64)
+    mu = q.mean(axis=0)
+    return mu, q.std(axis=0)
+
+
+def _build_proxies_no_gamma(qwin, z, gamma, t_len, dtype, rope_theta=0.0, rope_pos_offset=0):
+    mu, sigma = O.window_stats(qwin)
+    return O.round_to(mu[:, None, :] + sigma[:, None, :] * z, dtype)
+
+
+def _group_masses_wrong_gqa(proxies, keys, n_groups, scale):
+    hq, n_p, d = proxies.shape
+    t_len, hkv, _ = keys.shape
+    out = np.zeros((hkv, n_groups, t_len))
+    gs = n_p // n_groups
+    for h in range(hkv):
+        for g in range(n_groups):
+            rows = proxies[h::hkv, g * gs:(g + 1) * gs].reshape(-1, d)   # hq % Hkv mapping
+            out[h, g] = O.softmax_rows((rows @ keys[:, h].T) * scale).sum(axis=0)
+    return out
+
+
+_orig_group_masses = O.group_masses
+_orig_anchor = O.anchor_attention
+_orig_cover = O.cover_sets
+_orig_topk = O.select_topk
+_orig_normals = O.proxy_normals
+_orig_rope = O.rope_rotate
+_orig_philox = O.philox4x64_10
+
+
+def _group_masses_no_scale(proxies, keys, n_groups, scale):
+    return _orig_group_masses(proxies, keys, n_groups, 1.0)
+
+
+def _anchor_sum(q_last, keys, scale):
+    r = q_last.shape[0] // keys.shape[1]
+    return _orig_anchor(q_last, keys, scale) * r
+
+
+def _anchor_first_query(q_last, keys, scale):
+    # mistake planted in select_request's choice of query: use a different row
+    return _orig_anchor(q_last[::-1].copy(), keys, scale)
+
+
+def _cover_strict(abar, tau):
+    n_groups, t_len = abar.shape
+    member = np.zeros((n_groups, t_len), dtype=bool)
+    for g in range(n_groups):
+        order = np.lexsort((np.arange(t_len), -abar[g]))
+        csum = np.cumsum(abar[g][order])
+        k = int(np.argmax(csum > tau * csum[-1])) + 1
+        member[g, order[:k]] = True
+    return member
+
+
+def _topk_forgets_last(s, budget):
+    t_len = s.shape[0]
+    if budget >= t_len:
+        return np.arange(t_len)
+    order = np.lexsort((np.arange(t_len), -s))
+    return np.sort(order[:budget])
+
+
+def _topk_high_t_ties(s, budget):
+    t_len = s.shape[0]
+    if budget >= t_len:
+        return np.arange(t_len)
+    cand = np.arange(t_len - 1)
+    order = np.lexsort((-cand, -s[:t_len - 1]))
+    return np.sort(np.concatenate([order[:budget - 1], [t_len - 1]]))
+
+
+def _normals_no_two(seed, layer_id, b, n_q_heads, n_proxies, head_dim):
+    return _orig_normals(seed, layer_id, b, n_q_heads, n_proxies, head_dim) / math.sqrt(2.0)
+
+
+def _rope_wrong_sign(x, pos, theta):
+    return _orig_rope(x, -pos, theta)
+
+
+def _round_truncate(x, dtype):
+    x = np.asarray(x, dtype=np.float64)
+    if dtype == O.F32:
+        return x.astype(np.float32).astype(np.float64)
+    m, e = np.frexp(x)
+    ulp = np.ldexp(1.0, e - 8)
+    return np.trunc(x / ulp) * ulp
+
+
+def _philox_9_rounds(ctr, key):
+    c = [np.array(ctr[..., i], dtype=np.uint64) for i in range(4)]
+    k0, k1 = np.uint64(key[0]), np.uint64(key[1])
+    with np.errstate(over="ignore"):
+        for rnd in range(9):
+            if rnd:
+                k0 = np.uint64((int(k0) + int(O._PHILOX_W0)) & 0xFFFFFFFFFFFFFFFF)
+                k1 = np.uint64((int(k1) + int(O._PHILOX_W1)) & 0xFFFFFFFFFFFFFFFF)
+            hi0, lo0 = O._mulhilo64(c[0], O._PHILOX_M0)
+            hi1, lo1 = O._mulhilo64(c[2], O._PHILOX_M1)
+            c = [hi1 ^ c[1] ^ k0, lo1, hi0 ^ c[3] ^ k1, lo0]
+    return np.stack(c, axis=-1)
+
+
+MUTANTS = {
+    "std_ddof0": ("window_stats", _window_stats_ddof0),
+    "no_gamma": ("build_proxies", _build_proxies_no_gamma),
+    "gqa_modulo_mapping": ("group_masses", _group_masses_wrong_gqa),
+    "no_softmax_scale": ("group_masses", _group_masses_no_scale),
+    "anchor_sum_not_mean": ("anchor_attention", _anchor_sum),
+    "anchor_wrong_query": ("anchor_attention", _anchor_first_query),
+    "cover_strict_inequality": ("cover_sets", _cover_strict),
+    "topk_forgets_last_token": ("select_topk", _topk_forgets_last),
+    "topk_ties_high_t": ("select_topk", _topk_high_t_ties),
+    "box_muller_variance": ("proxy_normals", _normals_no_two),
+    "rope_sign": ("rope_rotate", _rope_wrong_sign),
+    "bf16_truncation": ("round_to", _round_truncate),
+    "philox_9_rounds": ("philox4x64_10", _philox_9_rounds),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_mutant_is_caught(name, monkeypatch):
+    attr, fn = MUTANTS[name]
+    monkeypatch.setattr(O, attr, fn)
+    caught = []
+    for pin in P.ALL_PINS:
+        try:
+            pin(O)
+        except Exception:
+            caught.append(pin.__name__)
+    assert caught, f"mutant {name} passed every pin"

@@ -1,0 +1,310 @@
+"""Pins of the CPU oracle against facts the paper and mathematics fix.
+
+None of these compare the oracle with itself: each check uses an independent
+library routine (numpy's Philox, scipy's softmax / distributions, Python's
+statistics module, torch's bf16 rounding), a closed form (Appendix A.2), an
+invariant (softmax rows sum to one, shift invariance, permutation
+equivariance) or exhaustive brute force on tiny inputs. ``test_oracle_mutants``
+plants plausible mistakes in the oracle and checks that these pins catch them.
+"""
+import itertools
+import json
+import math
+import os
+import statistics
+
+import numpy as np
+import pytest
+import scipy.special
+import scipy.stats
+
+from oracle import mmshift_oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+# ---------------------------------------------------------------------------
+# pin functions (shared with the mutant tests)
+# ---------------------------------------------------------------------------
+def pin_philox_vs_numpy(orc=O):
+    rng = np.random.default_rng(1)
+    for _ in range(20):
+        key = [int(x) for x in rng.integers(0, 2**63, size=2, dtype=np.uint64)]
+        ctr = [int(x) for x in rng.integers(0, 2**63, size=4, dtype=np.uint64)]
+        bg = np.random.Philox(key=key, counter=ctr)
+        ref = bg.random_raw(8)
+        # numpy advances the counter (low word first) before each block
+        c1 = np.array([[ctr[0] + 1, ctr[1], ctr[2], ctr[3]],
+                       [ctr[0] + 2, ctr[1], ctr[2], ctr[3]]], dtype=np.uint64)
+        got = orc.philox4x64_10(c1, key).reshape(-1)
+        np.testing.assert_array_equal(got, ref)
+
+
+def pin_normals_distribution(orc=O):
+    z = orc.proxy_normals(seed=7, layer_id=3, b=1, n_q_heads=4, n_proxies=4096, head_dim=64)
+    flat = z.reshape(-1)
+    n = flat.size
+    assert abs(flat.mean()) < 5.0 / math.sqrt(n)
+    assert abs(flat.var() - 1.0) < 5.0 * math.sqrt(2.0 / n)
+    ks = scipy.stats.kstest(flat[:200000], "norm")
+    assert ks.pvalue > 1e-4, ks
+    # the two normals of one Box-Muller pair are uncorrelated
+    pair = z.reshape(-1, 2)
+    corr = np.corrcoef(pair[:, 0], pair[:, 1])[0, 1]
+    assert abs(corr) < 5.0 / math.sqrt(pair.shape[0])
+    # distinct counters (heads, requests, layers, seeds) give distinct streams
+    z2 = orc.proxy_normals(seed=7, layer_id=4, b=1, n_q_heads=4, n_proxies=64, head_dim=64)
+    assert not np.allclose(z[:, :64], z2)
+
+
+def pin_window_stats(orc=O):
+    rng = np.random.default_rng(2)
+    q = rng.normal(size=(9, 3, 5)) * 3.0 + 1.0
+    mu, sigma = orc.window_stats(q)
+    for h in range(3):
+        for j in range(5):
+            col = [float(v) for v in q[:, h, j]]
+            assert math.isclose(mu[h, j], statistics.fmean(col), rel_tol=1e-12, abs_tol=1e-12)
+            assert math.isclose(sigma[h, j], statistics.stdev(col), rel_tol=1e-12)
+
+
+def pin_sampler_closed_form(orc=O):
+    """Appendix A.2: for q ~ N(mu, Sigma), E[exp(q.k/sqrt d)] =
+    exp(mu.k/sqrt d + k^T Sigma k / (2d)). With Sigma = diag((gamma*sigma)^2)
+    the proxies' Monte-Carlo mean must match within its CLT band."""
+    rng = np.random.default_rng(3)
+    d, w, n_p = 16, 8, 1 << 16
+    qwin = rng.normal(size=(w, 1, d)) * 0.3 + 0.2
+    z = orc.proxy_normals(seed=11, layer_id=0, b=0, n_q_heads=1, n_proxies=n_p, head_dim=d)
+    gamma = 2.0
+    prox = orc.build_proxies(qwin, z, gamma, t_len=100, dtype=orc.F32)[0]   # [Np, d]
+    mu = qwin[:, 0, :].mean(axis=0)
+    sig = qwin[:, 0, :].std(axis=0, ddof=1)
+    # per-dimension moments of the proxies: mean mu, std gamma*sigma
+    np.testing.assert_allclose(prox.mean(axis=0), mu, atol=6.0 * gamma * sig.max() / math.sqrt(n_p))
+    np.testing.assert_allclose(prox.std(axis=0), gamma * sig, rtol=6.0 / math.sqrt(2 * n_p))
+    for _ in range(4):
+        k = rng.normal(size=d) * 0.5
+        e = np.exp(prox @ k / math.sqrt(d))
+        closed = math.exp(mu @ k / math.sqrt(d) + np.sum((gamma * sig) ** 2 * k ** 2) / (2 * d))
+        se = e.std() / math.sqrt(n_p)
+        assert abs(e.mean() - closed) < 6.0 * se, (e.mean(), closed, se)
+
+
+def pin_rope(orc=O):
+    rng = np.random.default_rng(4)
+    d, theta = 16, 10000.0
+    x = rng.normal(size=(3, d))
+    pos = 37.0
+    got = orc.rope_rotate(x, pos, theta)
+    half = d // 2
+    zc = (x[:, :half] + 1j * x[:, half:]) * np.exp(1j * pos * theta ** (-2.0 * np.arange(half) / d))
+    np.testing.assert_allclose(got, np.concatenate([zc.real, zc.imag], axis=1), atol=1e-12)
+    np.testing.assert_allclose(np.linalg.norm(got, axis=1), np.linalg.norm(x, axis=1), rtol=1e-12)
+    # relative-position property: <R_m q, R_n k> depends on m - n only
+    q, k = x[0], x[1]
+    a = orc.rope_rotate(q, 50.0, theta) @ orc.rope_rotate(k, 20.0, theta)
+    b = orc.rope_rotate(q, 130.0, theta) @ orc.rope_rotate(k, 100.0, theta)
+    assert math.isclose(a, b, rel_tol=1e-9, abs_tol=1e-12)
+
+
+def pin_round_bf16(orc=O):
+    import torch
+    rng = np.random.default_rng(5)
+    x = (rng.normal(size=20000) * 10.0 ** rng.uniform(-6, 6, size=20000)).astype(np.float32)
+    ref = torch.from_numpy(x).to(torch.bfloat16).to(torch.float64).numpy()
+    np.testing.assert_array_equal(orc.round_to(x.astype(np.float64), orc.BF16), ref)
+    # exact halfway cases go to the even neighbour
+    one = 1.0
+    ulp = 2.0 ** -7
+    halfway = np.array([one + ulp / 2, one + 3 * ulp / 2, -(one + ulp / 2)])
+    np.testing.assert_array_equal(orc.round_to(halfway, orc.BF16),
+                                  np.array([one, one + 2 * ulp, -one]))
+
+
+def _tiny_problem(seed, t_len=40, hq=4, hkv=2, d=8, n_p=8, scale_k=1.0):
+    rng = np.random.default_rng(seed)
+    keys = rng.normal(size=(t_len, hkv, d)) * scale_k
+    proxies = rng.normal(size=(hq, n_p, d)) * 2.0
+    q_last = rng.normal(size=(hq, d))
+    return keys, proxies, q_last
+
+
+def pin_mass_totals(orc=O):
+    keys, proxies, q_last = _tiny_problem(6)
+    hq, n_p, d = proxies.shape
+    hkv = keys.shape[1]
+    r = hq // hkv
+    scale = 1.0 / math.sqrt(d)
+    a = orc.softmax_rows(rng_logits := np.random.default_rng(6).normal(size=(5, 30)) * 20)
+    np.testing.assert_allclose(a.sum(axis=1), 1.0, atol=1e-12)
+    np.testing.assert_allclose(a, scipy.special.softmax(rng_logits, axis=1), rtol=1e-12, atol=1e-300)
+    for n_groups in (1, 2, 4, 8):
+        abar = orc.group_masses(proxies, keys, n_groups, scale)
+        gs = n_p // n_groups
+        np.testing.assert_allclose(abar.sum(axis=2), gs * r, rtol=1e-12)
+        np.testing.assert_allclose(abar.sum(axis=(1, 2)), n_p * r, rtol=1e-12)
+    alpha = orc.anchor_attention(q_last, keys, scale)
+    np.testing.assert_allclose(alpha.sum(axis=1), 1.0, rtol=1e-12)
+
+
+def pin_sigma_zero_single_query(orc=O):
+    """Identical window queries: sigma = 0, every proxy equals mu, and each
+    group mass is gs * (sum over the r heads of) one softmax row."""
+    rng = np.random.default_rng(7)
+    t_len, hq, hkv, d, w, n_p, n_groups = 50, 6, 2, 8, 5, 8, 2
+    r = hq // hkv
+    keys = rng.normal(size=(t_len, hkv, d))
+    qrow = rng.normal(size=(hq, d))
+    qwin = np.repeat(qrow[None], w, axis=0)
+    z = rng.normal(size=(hq, n_p, d))
+    prox = orc.build_proxies(qwin, z, 10.0, t_len, orc.F32)
+    np.testing.assert_allclose(prox, np.broadcast_to(orc.round_to(qrow, orc.F32)[:, None, :], prox.shape))
+    abar = orc.group_masses(prox, keys, n_groups, 1.0 / math.sqrt(d))
+    gs = n_p // n_groups
+    for h in range(hkv):
+        heads = [hh for hh in range(hq) if hh // r == h]
+        expect = sum(scipy.special.softmax(prox[hh, 0] @ keys[:, h, :].T / math.sqrt(d)) for hh in heads) * gs
+        for g in range(n_groups):
+            np.testing.assert_allclose(abar[h, g], expect, rtol=1e-10)
+
+
+def pin_shift_and_permutation(orc=O):
+    keys, proxies, q_last = _tiny_problem(8, t_len=30)
+    t_len, hkv, d = keys.shape
+    hq = proxies.shape[0]
+    qwin = np.concatenate([np.random.default_rng(9).normal(size=(3, hq, d)), q_last[None]], axis=0)
+    kw = dict(n_proxies=proxies.shape[1], n_groups=2, proxies=proxies, dtype=orc.F32, tau=0.9)
+    base = orc.select_request(keys, keys, qwin, 12, **kw)
+    # same vector added to every key of a head: every softmax row is unchanged
+    u = np.random.default_rng(10).normal(size=(1, hkv, d)) * 3.0
+    sh = orc.select_request(keys + u, keys, qwin, 12, **kw)
+    np.testing.assert_allclose(sh["group_mass"], base["group_mass"], rtol=1e-9, atol=1e-300)
+    np.testing.assert_allclose(sh["anchor"], base["anchor"], rtol=1e-9, atol=1e-300)
+    np.testing.assert_array_equal(sh["idx"], base["idx"])
+    # permuting the keys permutes masses and scores
+    perm = np.random.default_rng(11).permutation(t_len - 1)
+    perm = np.concatenate([perm, [t_len - 1]])
+    pm = orc.select_request(keys[perm], keys[perm], qwin, 12, **kw)
+    np.testing.assert_allclose(pm["group_mass"], base["group_mass"][:, :, perm], rtol=1e-9, atol=1e-300)
+    np.testing.assert_allclose(pm["scores"], base["scores"][:, perm], rtol=1e-9, atol=1e-300)
+    for h in range(hkv):
+        assert set(perm[pm["idx"][:, h]]) == set(base["idx"][:, h])
+
+
+def pin_budget_ge_t(orc=O):
+    keys, proxies, q_last = _tiny_problem(12, t_len=17)
+    qwin = np.stack([q_last, q_last * 0.5, q_last], axis=0)
+    for budget in (17, 18, 1000):
+        res = orc.select_request(keys, keys, qwin, budget, n_proxies=8, n_groups=4,
+                                 proxies=proxies, dtype=orc.F32)
+        for h in range(keys.shape[1]):
+            np.testing.assert_array_equal(res["idx"][:, h], np.arange(17))
+    res = orc.select_request(keys, keys, qwin, 1, n_proxies=8, n_groups=4, proxies=proxies,
+                             dtype=orc.F32)
+    np.testing.assert_array_equal(res["idx"], np.full((1, keys.shape[1]), 16))
+
+
+def pin_lastattn(orc=O):
+    """tau = 1 puts every key with positive mass in every cover set, so all
+    votes tie at G and the ranking is the last query's attention alone (the
+    'LastAttn' row of Table 5)."""
+    rng = np.random.default_rng(13)
+    t_len, hq, hkv, d = 60, 4, 2, 8
+    r = hq // hkv
+    keys = rng.normal(size=(t_len, hkv, d))
+    qwin = rng.normal(size=(4, hq, d))
+    proxies = rng.normal(size=(hq, 8, d))
+    budget = 20
+    res = orc.select_request(keys, keys, qwin, budget, n_proxies=8, n_groups=4, tau=1.0,
+                             proxies=proxies, dtype=orc.F32)
+    assert np.all(res["scores"] >= 4.0)
+    for h in range(hkv):
+        heads = [hh for hh in range(hq) if hh // r == h]
+        att = np.mean([scipy.special.softmax(qwin[-1, hh] @ keys[:, h].T / math.sqrt(d)) for hh in heads], axis=0)
+        np.testing.assert_allclose(res["anchor"][h], att, rtol=1e-12)
+        top = np.argsort(-att[:t_len - 1], kind="stable")[:budget - 1]
+        np.testing.assert_array_equal(res["idx"][:, h], np.sort(np.concatenate([top, [t_len - 1]])))
+
+
+def pin_uniform_keys(orc=O):
+    t_len, d = 100, 8
+    keys = np.ones((t_len, 1, d))
+    proxies = np.random.default_rng(14).normal(size=(2, 8, d))
+    abar = orc.group_masses(proxies, keys, 2, 1.0 / math.sqrt(d))
+    assert np.all(abar == abar[:, :, :1])
+    member = orc.cover_sets(abar[0], 0.955)
+    for g in range(2):
+        np.testing.assert_array_equal(np.nonzero(member[g])[0], np.arange(96))
+
+
+def _brute_cover(mass, tau):
+    t_len = mass.size
+    total = mass.sum()
+    for size in range(0, t_len + 1):
+        ok = [set(c) for c in itertools.combinations(range(t_len), size)
+              if mass[list(c)].sum() >= tau * total - 1e-12]
+        if ok:
+            return size, ok
+    raise AssertionError
+
+
+def pin_cover_bruteforce(orc=O):
+    rng = np.random.default_rng(15)
+    for trial in range(60):
+        t_len = int(rng.integers(1, 10))
+        mass = rng.integers(0, 5, size=(2, t_len)).astype(np.float64)
+        mass[:, 0] += 1.0                         # no all-zero group
+        tau = float(rng.choice([0.3, 0.5, 0.7, 0.9, 1.0]))
+        member = orc.cover_sets(mass, tau)
+        for g in range(2):
+            chosen = set(np.nonzero(member[g])[0].tolist())
+            size, ok = _brute_cover(mass[g], tau)
+            assert len(chosen) == size, (mass[g], tau, chosen, size)
+            assert chosen in ok
+            # prefix of the (mass desc, t asc) ranking
+            for t in chosen:
+                for u in set(range(t_len)) - chosen:
+                    assert mass[g, t] > mass[g, u] or (mass[g, t] == mass[g, u] and t < u)
+
+
+def pin_topk_bruteforce(orc=O):
+    rng = np.random.default_rng(16)
+    for trial in range(80):
+        t_len = int(rng.integers(1, 10))
+        s = rng.integers(0, 4, size=t_len).astype(np.float64) + 0.25 * rng.integers(0, 2, size=t_len)
+        for budget in range(1, t_len + 2):
+            got = orc.select_topk(s, budget)
+            if budget >= t_len:
+                np.testing.assert_array_equal(got, np.arange(t_len))
+                continue
+            assert got[-1] == t_len - 1 and np.all(np.diff(got) > 0)
+            cand = [int(t) for t in got[:-1]]
+            best = max(sum(s[list(c)]) for c in itertools.combinations(range(t_len - 1), budget - 1))
+            assert math.isclose(sum(s[cand]), best)
+            # among the best sets the lowest indices win ties
+            bests = sorted(sorted(c) for c in itertools.combinations(range(t_len - 1), budget - 1)
+                           if math.isclose(sum(s[list(c)]), best))
+            assert cand == list(bests[0])
+
+
+ALL_PINS = [pin_philox_vs_numpy, pin_normals_distribution, pin_window_stats,
+            pin_sampler_closed_form, pin_rope, pin_round_bf16, pin_mass_totals,
+            pin_sigma_zero_single_query, pin_shift_and_permutation, pin_budget_ge_t,
+            pin_lastattn, pin_uniform_keys, pin_cover_bruteforce, pin_topk_bruteforce]
+
+
+@pytest.mark.parametrize("pin", ALL_PINS, ids=[p.__name__ for p in ALL_PINS])
+def test_pin(pin):
+    pin()
+
+
+def test_defaults_match_paper():
+    with open(os.path.join(GOLDEN, "hyperparams.json")) as f:
+        g = json.load(f)
+    assert O.DEFAULTS["n_proxies"] == g["n_proxies"]
+    assert O.DEFAULTS["n_groups"] == g["n_groups"]
+    assert g["n_proxies"] // g["n_groups"] == g["group_size"]
+    assert O.DEFAULTS["gamma"] == g["gamma"]
+    assert O.DEFAULTS["tau"] == g["tau"]
+    assert O.DEFAULTS["lam"] == g["lambda"]
