@@ -1,0 +1,204 @@
+/*
+ * mmshift.h -- C ABI of the GB300 (sm_103a) prefill-only KV selection library.
+ *
+ * The library implements MM-ShiftKV's selection step (the paper's Section 3.2
+ * and Algorithm 1 in Appendix B): after prefill, for every layer and KV head,
+ *   1. build variance-expanded query proxies from the observation-window
+ *      queries (Section 3.2.1, Appendix A.4);
+ *   2. score every prompt key with the proxies' attention logits under GQA
+ *      head grouping, 3. softmax over the whole prompt (Section 3.2.2);
+ *   4. aggregate the attention mass per proxy group and vote with the
+ *      tau-coverage rule, add the last-query anchor (Sections 3.2.2-3.2.3);
+ *   5. keep the last token plus the top C-1 keys (Section 3.2.3);
+ *   6. gather the kept K/V rows, in temporal order, into a compact cache
+ *      (Appendix B).
+ *
+ * Conventions shared by every entry point:
+ *   - All pointers except the ones marked "host" are device pointers. The
+ *     caller owns every buffer; the library allocates no device memory and,
+ *     apart from mmshift_poll_status, never synchronises.
+ *   - All work is enqueued on `stream` (a cudaStream_t; NULL is the legacy
+ *     default stream) and is asynchronous.
+ *   - Host-side validation runs first; on error nothing is enqueued and the
+ *     outputs are untouched. Errors from the CUDA runtime are returned as
+ *     MMSHIFT_ERR_CUDA (see mmshift_last_cuda_error).
+ *   - Token data is "varlen packed": requests are concatenated along the token
+ *     axis with host prefix offsets cu_seqlens[0..batch] (cu_seqlens[0] = 0).
+ *   - A call covers n_layers layers; layer l reads K + l*layer_stride_kv,
+ *     V + l*layer_stride_kv and Qwin + l*layer_stride_q (strides in elements)
+ *     and uses the random-stream layer id params.layer_id + l. Every output
+ *     and debug buffer is laid out [n_layers, ...] contiguously.
+ *   - Results are deterministic for fixed inputs and (seed, layer_id).
+ *
+ * Shapes (T = total tokens = cu_seqlens[batch], R = sum_b min(C_b, T_b)):
+ *   K, V        [T, Hkv, d]        dtype; rows contiguous (d elements)
+ *   Qwin        [batch, W, Hq, d]  dtype; the W last prefill queries of each
+ *                                  request, the last row being the last real
+ *                                  prefill query (the anchor of Section 3.2.3)
+ *   proxies     [batch, Hq, N, d]  dtype
+ *   group_mass  [Hkv, G, T]        float32  (per layer)
+ *   anchor, mass, scores [Hkv, T]  float32  (per layer)
+ *   out_idx     [R, Hkv]           int32 token index within its request;
+ *                                  request b owns rows [sum_{b'<b} C'_b', +C'_b),
+ *                                  ascending in each column (temporal order)
+ *   out_K/out_V [R, Hkv, d]        dtype; out_K[c, h] = K[cu_b + out_idx[c, h], h]
+ */
+#ifndef MMSHIFT_H
+#define MMSHIFT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* mmshift_stream_t; /* same type as cudaStream_t */
+
+typedef enum {
+  MMSHIFT_OK = 0,
+  MMSHIFT_ERR_INVALID_ARG = 1, /* null pointer, bad shape, bad parameter */
+  MMSHIFT_ERR_UNSUPPORTED = 2, /* valid but not implemented (dtype, head_dim) */
+  MMSHIFT_ERR_WORKSPACE = 3,   /* workspace missing, too small or misaligned */
+  MMSHIFT_ERR_CUDA = 4,        /* a CUDA runtime call failed */
+  MMSHIFT_ERR_TIMEOUT = 5,     /* a bounded device-side wait gave up */
+  MMSHIFT_ERR_DEVICE = 6       /* a device-side check failed */
+} mmshift_status;
+
+enum { MMSHIFT_BF16 = 0, MMSHIFT_F32 = 1 };
+
+/* Importance score used by the budgeted top-k.
+ * VOTE: S_t = vote(t) + lambda * anchor_t (Sections 3.2.2-3.2.3; the paper's
+ *       method). MASS: S_t = sum_g group_mass[g, t] (the Table 5 ablation row
+ *       with sampling and variance expansion but no group vote). */
+enum { MMSHIFT_SCORE_VOTE = 0, MMSHIFT_SCORE_MASS = 1 };
+
+#define MMSHIFT_MAX_BATCH 64
+#define MMSHIFT_MAX_LAYERS 4096
+
+/* Method hyper-parameters; defaults (mmshift_default_params) are the paper's
+ * Section 4.1 values: N = 512 proxies in G = 32 groups, gamma = 10,
+ * tau = 0.95, lambda = 1. */
+typedef struct {
+  int32_t n_proxies;      /* N per query head; 0 with n_groups = 0 = anchor only */
+  int32_t n_groups;       /* G; n_proxies % n_groups == 0 */
+  float gamma;            /* variance expansion, > 0 (Section 3.2.1) */
+  float tau;              /* coverage threshold, 0 < tau <= 1 (Section 3.2.2) */
+  float lambda;           /* anchor weight, >= 0 (Section 3.2.3) */
+  int32_t score_mode;     /* MMSHIFT_SCORE_VOTE or MMSHIFT_SCORE_MASS */
+  uint64_t seed;          /* key of the proxy random stream */
+  int32_t layer_id;       /* layer id of the first layer of the call */
+  float softmax_scale;    /* 0 => 1/sqrt(head_dim) */
+  float rope_theta;       /* > 0 rotates proxies (RoPE base); 0 => no RoPE */
+  int32_t rope_pos_offset;/* proxies sit at position T_b + rope_pos_offset */
+} mmshift_params;
+
+typedef struct {
+  int32_t batch;            /* 1..MMSHIFT_MAX_BATCH requests */
+  int32_t n_q_heads;        /* Hq, multiple of n_kv_heads */
+  int32_t n_kv_heads;       /* Hkv */
+  int32_t head_dim;         /* d: 64 or 128 */
+  int32_t window;           /* W >= 2 observation-window queries */
+  int32_t dtype;            /* MMSHIFT_BF16 or MMSHIFT_F32 */
+  const int32_t* cu_seqlens;/* host [batch+1], T_b = cu[b+1]-cu[b] >= 1 */
+  const int32_t* budgets;   /* host [batch], C_b >= 1 */
+  int32_t n_layers;         /* 1..MMSHIFT_MAX_LAYERS */
+  int64_t layer_stride_kv;  /* elements between layers of K and V (>= T*Hkv*d) */
+  int64_t layer_stride_q;   /* elements between layers of Qwin (>= B*W*Hq*d) */
+} mmshift_shape;
+
+/* Optional intermediate outputs of mmshift_select (any may be NULL). */
+typedef struct {
+  void* proxies;     /* [L, batch, Hq, N, d] dtype: the sampled proxies */
+  float* group_mass; /* [L, Hkv, G, T] attention mass of each proxy group */
+  float* anchor;     /* [L, Hkv, T] last-query attention, mean over the GQA heads */
+  float* mass;       /* [L, Hkv, T] sum_g group_mass */
+  float* scores;     /* [L, Hkv, T] S_t used by the top-k */
+} mmshift_debug;
+
+/* Fill *p with the paper's default hyper-parameters (Section 4.1). */
+void mmshift_default_params(mmshift_params* p);
+
+/* Rows R = sum_b min(C_b, T_b) of out_idx / out_K / out_V per layer. */
+mmshift_status mmshift_output_rows(const mmshift_shape* s, int64_t* rows);
+
+/* Bytes of device workspace the calls below need for (s, p); 256-byte
+ * alignment is required. The same workspace serves every entry point. */
+mmshift_status mmshift_workspace_size(const mmshift_shape* s, const mmshift_params* p,
+                                      size_t* bytes);
+
+/* Step 1 alone (Section 3.2.1, Appendix A.4): per (request, query head,
+ * dimension) mean and unbiased std over the W window queries, then
+ * proxies[b, hq, i, j] = mu + gamma * sigma * z with z ~ N(0, 1) drawn from
+ * Philox4x64-10 + Box-Muller (counter (i*d/4 + j/4, hq, b, layer_id), key
+ * (seed, 0)), optionally RoPE-rotated to position T_b + rope_pos_offset, and
+ * rounded to dtype. proxies: [L, batch, Hq, N, d]. */
+mmshift_status mmshift_build_proxies(const mmshift_shape* s, const void* Qwin,
+                                     const mmshift_params* p, void* proxies,
+                                     mmshift_stream_t stream);
+
+/* Steps 2-4 (Section 3.2.2, Appendix B): softmax attention of every proxy over
+ * all T_b keys of its KV head (h = hq / r), summed per proxy group over the r
+ * query heads of that KV head; and the last-query anchor (mean over the r
+ * heads). `proxies` ([L, batch, Hq, N, d]) may be NULL, in which case they
+ * are sampled as in mmshift_build_proxies. Outputs are [L, ...] float32;
+ * `mass` may be NULL. */
+mmshift_status mmshift_proxy_mass(const mmshift_shape* s, const void* K, const void* Qwin,
+                                  const void* proxies, const mmshift_params* p,
+                                  float* group_mass, float* anchor, float* mass,
+                                  void* workspace, size_t workspace_bytes,
+                                  mmshift_stream_t stream);
+
+/* Step 5 from masses (Sections 3.2.2-3.2.3): tau-coverage sets per (KV head,
+ * group) -- the smallest prefix of keys by descending mass (ties: lower t
+ * first) holding at least tau of the group's mass --, votes, S_t = vote +
+ * lambda * anchor (or sum_g mass in MASS mode), then the kept indices.
+ * group_mass [L, Hkv, G, T], anchor [L, Hkv, T] (unused in MASS mode);
+ * scores (nullable) [L, Hkv, T]; out_idx [L, R, Hkv]. */
+mmshift_status mmshift_scores_topk(const mmshift_shape* s, const mmshift_params* p,
+                                   const float* group_mass, const float* anchor,
+                                   float* scores, int32_t* out_idx,
+                                   void* workspace, size_t workspace_bytes,
+                                   mmshift_stream_t stream);
+
+/* Budgeted selection from given scores (Section 3.2.3): token T_b-1 always,
+ * plus the C_b-1 largest S_t among t < T_b-1 (ties: lower t first), in
+ * ascending order; C_b >= T_b keeps every token. scores [L, Hkv, T] float32,
+ * finite; out_idx [L, R, Hkv]. */
+mmshift_status mmshift_topk(const mmshift_shape* s, const float* scores, int32_t* out_idx,
+                            void* workspace, size_t workspace_bytes,
+                            mmshift_stream_t stream);
+
+/* Step 6 (Appendix B): out_K[c, h] = K[cu_b + idx[c, h], h], same for V; a
+ * bit copy. idx [L, R, Hkv] must hold indices in [0, T_b); out of range rows
+ * are zero-filled and reported by mmshift_poll_status. */
+mmshift_status mmshift_gather(const mmshift_shape* s, const void* K, const void* V,
+                              const int32_t* idx, void* out_K, void* out_V,
+                              void* workspace, size_t workspace_bytes,
+                              mmshift_stream_t stream);
+
+/* The whole selection (Algorithm 1): steps 1-6 for L layers. `proxies_in`
+ * (nullable, [L, batch, Hq, N, d]) replaces the sampled proxies, e.g. for
+ * proxies a caller projects from hidden states. `dbg` (nullable) receives
+ * intermediate results. */
+mmshift_status mmshift_select(const mmshift_shape* s, const void* K, const void* V,
+                              const void* Qwin, const void* proxies_in,
+                              const mmshift_params* p, int32_t* out_idx, void* out_K,
+                              void* out_V, const mmshift_debug* dbg, void* workspace,
+                              size_t workspace_bytes, mmshift_stream_t stream);
+
+/* Synchronise `stream`, read and clear the device status word kept in the
+ * workspace: MMSHIFT_OK, MMSHIFT_ERR_TIMEOUT or MMSHIFT_ERR_DEVICE. */
+mmshift_status mmshift_poll_status(void* workspace, mmshift_stream_t stream);
+
+/* Human-readable name of a status code. */
+const char* mmshift_status_string(mmshift_status st);
+
+/* Text of the last CUDA runtime error seen on this host thread ("" if none). */
+const char* mmshift_last_cuda_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MMSHIFT_H */

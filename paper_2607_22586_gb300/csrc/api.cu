@@ -1,0 +1,367 @@
+// Host side of the C ABI declared in include/mmshift.h: argument validation,
+// problem description, workspace carve-up and kernel sequencing. Nothing here
+// allocates device memory or synchronises (except mmshift_poll_status).
+#include <cmath>
+#include <cstring>
+#include <string>
+
+#include "common.cuh"
+
+using namespace mmshift;
+
+namespace {
+
+thread_local std::string g_cuda_error;
+
+mmshift_status cuda_fail(cudaError_t e) {
+  g_cuda_error = cudaGetErrorString(e);
+  return MMSHIFT_ERR_CUDA;
+}
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+int roundup(int x, int m) { return (x + m - 1) / m * m; }
+
+mmshift_status check_shape(const mmshift_shape* s) {
+  if (!s || !s->cu_seqlens || !s->budgets) return MMSHIFT_ERR_INVALID_ARG;
+  if (s->batch < 1 || s->batch > MMSHIFT_MAX_BATCH) return MMSHIFT_ERR_INVALID_ARG;
+  if (s->n_layers < 1 || s->n_layers > MMSHIFT_MAX_LAYERS) return MMSHIFT_ERR_INVALID_ARG;
+  if (s->n_kv_heads < 1 || s->n_q_heads < s->n_kv_heads || s->n_q_heads % s->n_kv_heads)
+    return MMSHIFT_ERR_INVALID_ARG;
+  if (s->window < 2) return MMSHIFT_ERR_INVALID_ARG;
+  if (s->dtype != MMSHIFT_BF16 && s->dtype != MMSHIFT_F32) return MMSHIFT_ERR_UNSUPPORTED;
+  if (s->head_dim != 64 && s->head_dim != 128) return MMSHIFT_ERR_UNSUPPORTED;
+  if (s->cu_seqlens[0] != 0) return MMSHIFT_ERR_INVALID_ARG;
+  int64_t total = 0;
+  for (int b = 0; b < s->batch; ++b) {
+    const int64_t t = (int64_t)s->cu_seqlens[b + 1] - s->cu_seqlens[b];
+    if (t < 1 || s->budgets[b] < 1) return MMSHIFT_ERR_INVALID_ARG;
+    total += t;
+  }
+  if (total > (int64_t)1 << 30) return MMSHIFT_ERR_UNSUPPORTED;
+  if (s->n_layers > 1) {
+    if (s->layer_stride_kv < total * s->n_kv_heads * s->head_dim) return MMSHIFT_ERR_INVALID_ARG;
+    if (s->layer_stride_q < (int64_t)s->batch * s->window * s->n_q_heads * s->head_dim)
+      return MMSHIFT_ERR_INVALID_ARG;
+  }
+  return MMSHIFT_OK;
+}
+
+mmshift_status check_params(const mmshift_params* p) {
+  if (!p) return MMSHIFT_ERR_INVALID_ARG;
+  if (p->n_proxies < 0 || p->n_groups < 0) return MMSHIFT_ERR_INVALID_ARG;
+  if ((p->n_proxies == 0) != (p->n_groups == 0)) return MMSHIFT_ERR_INVALID_ARG;
+  if (p->n_groups && p->n_proxies % p->n_groups) return MMSHIFT_ERR_INVALID_ARG;
+  if (p->n_groups > 1024) return MMSHIFT_ERR_UNSUPPORTED;
+  if (!(p->gamma > 0.f) || !std::isfinite(p->gamma)) return MMSHIFT_ERR_INVALID_ARG;
+  if (!(p->tau > 0.f) || p->tau > 1.f) return MMSHIFT_ERR_INVALID_ARG;
+  if (!(p->lambda >= 0.f) || !std::isfinite(p->lambda)) return MMSHIFT_ERR_INVALID_ARG;
+  if (p->score_mode != MMSHIFT_SCORE_VOTE && p->score_mode != MMSHIFT_SCORE_MASS)
+    return MMSHIFT_ERR_INVALID_ARG;
+  if (!(p->softmax_scale >= 0.f) || !std::isfinite(p->softmax_scale)) return MMSHIFT_ERR_INVALID_ARG;
+  if (!(p->rope_theta >= 0.f) || !std::isfinite(p->rope_theta)) return MMSHIFT_ERR_INVALID_ARG;
+  if (p->layer_id < 0) return MMSHIFT_ERR_INVALID_ARG;
+  return MMSHIFT_OK;
+}
+
+// Key split length of the softmax pass. It is a constant, so the order in
+// which a request's partial (max, sum) pairs are merged -- and with it every
+// bit of the result -- does not depend on the other requests or layers of the
+// call.
+constexpr int kSplitLen = 1024;
+
+mmshift_status build_problem(const mmshift_shape* s, const mmshift_params* p, Problem* P) {
+  std::memset(P, 0, sizeof(*P));
+  P->B = s->batch;
+  P->L = s->n_layers;
+  P->Hq = s->n_q_heads;
+  P->Hkv = s->n_kv_heads;
+  P->r = s->n_q_heads / s->n_kv_heads;
+  P->d = s->head_dim;
+  P->W = s->window;
+  P->dtype = s->dtype;
+  P->Np = p->n_proxies;
+  P->G = p->n_groups;
+  P->gs = P->G ? P->Np / P->G : 0;
+  P->RG = roundup(P->r * P->gs, kChunk);
+  P->n_group_rows = P->G * P->RG;
+  P->anchor_rows = roundup(P->r, kChunk);
+  P->Prows = P->n_group_rows + P->anchor_rows;
+  P->Prows_pad = roundup(P->Prows, kRowTile);
+  int64_t tot = 0, outr = 0, words = 0;
+  for (int b = 0; b < P->B; ++b) {
+    ReqInfo& R = P->req[b];
+    R.t_len = s->cu_seqlens[b + 1] - s->cu_seqlens[b];
+    R.tok_off = s->cu_seqlens[b];
+    R.budget = s->budgets[b];
+    R.keep = std::min(R.budget, R.t_len);
+    R.out_off = (int32_t)outr;
+    R.word_off = (int32_t)words;
+    tot += R.t_len;
+    outr += R.keep;
+    words += (R.t_len + 31) / 32;
+  }
+  P->total_T = (int32_t)tot;
+  P->R = (int32_t)outr;
+  P->total_words = (int32_t)words;
+  P->ls_kv = s->n_layers > 1 ? s->layer_stride_kv : 0;
+  P->ls_q = s->n_layers > 1 ? s->layer_stride_q : 0;
+  P->scale = p->softmax_scale > 0.f ? p->softmax_scale : 1.0f / std::sqrt((float)s->head_dim);
+  P->alpha = P->scale * kLog2e;
+  P->gamma = p->gamma;
+  P->tau = p->tau;
+  P->lambda = p->lambda;
+  P->mode = p->score_mode;
+  P->seed = p->seed;
+  P->layer_id0 = p->layer_id;
+  P->rope_theta = p->rope_theta;
+  P->rope_off = p->rope_pos_offset;
+  P->split_len = kSplitLen;
+  int32_t so = 0;
+  for (int b = 0; b < P->B; ++b) {
+    ReqInfo& R = P->req[b];
+    R.nsplit = (R.t_len + P->split_len - 1) / P->split_len;
+    R.split_off = so;
+    so += R.nsplit;
+  }
+  P->total_splits = so;
+  return MMSHIFT_OK;
+}
+
+struct Layout {
+  size_t status, packed, part, cvals, gmass, anchor, bits, scores, total;
+};
+
+Layout layout_of(const Problem& P) {
+  const size_t esz = P.dtype == MMSHIFT_BF16 ? 2 : 4;
+  const size_t L = P.L;
+  Layout w;
+  size_t o = 0;
+  w.status = o; o += 256;
+  w.packed = o; o += align256(L * P.B * P.Hkv * (size_t)P.Prows_pad * P.d * esz);
+  w.part = o;   o += align256(L * P.Hkv * (size_t)P.total_splits * P.Prows_pad * sizeof(float2));
+  w.cvals = o;  o += align256(L * P.B * P.Hkv * (size_t)P.Prows_pad * sizeof(float));
+  w.gmass = o;  o += align256(L * P.Hkv * (size_t)P.G * P.total_T * sizeof(float));
+  w.anchor = o; o += align256(L * P.Hkv * (size_t)P.total_T * sizeof(float));
+  w.bits = o;   o += align256(L * P.Hkv * (size_t)P.G * P.total_words * sizeof(uint32_t));
+  w.scores = o; o += align256(L * P.Hkv * (size_t)P.total_T * sizeof(float));
+  w.total = o;
+  return w;
+}
+
+mmshift_status carve(const Problem& P, void* ws, size_t bytes, Buffers* bf) {
+  const Layout w = layout_of(P);
+  if (!ws || bytes < w.total) return MMSHIFT_ERR_WORKSPACE;
+  if (reinterpret_cast<uintptr_t>(ws) & 255) return MMSHIFT_ERR_WORKSPACE;
+  char* base = static_cast<char*>(ws);
+  std::memset(bf, 0, sizeof(*bf));
+  bf->status = reinterpret_cast<int*>(base + w.status);
+  bf->packed = base + w.packed;
+  bf->part = reinterpret_cast<float2*>(base + w.part);
+  bf->cvals = reinterpret_cast<float*>(base + w.cvals);
+  bf->gmass = reinterpret_cast<float*>(base + w.gmass);
+  bf->anchor = reinterpret_cast<float*>(base + w.anchor);
+  bf->bits = reinterpret_cast<uint32_t*>(base + w.bits);
+  bf->scores = reinterpret_cast<float*>(base + w.scores);
+  return MMSHIFT_OK;
+}
+
+mmshift_status prepare(const mmshift_shape* s, const mmshift_params* p, Problem* P) {
+  mmshift_status st = check_shape(s);
+  if (st != MMSHIFT_OK) return st;
+  mmshift_params dflt;
+  if (!p) { mmshift_default_params(&dflt); p = &dflt; }
+  if ((st = check_params(p)) != MMSHIFT_OK) return st;
+  return build_problem(s, p, P);
+}
+
+// Proxies (sampled or given) packed into the workspace, then steps 2-4.
+mmshift_status run_mass(const Problem& P, const Buffers& bf, const void* K, const void* qwin,
+                        cudaStream_t st) {
+  cudaError_t e = launch_proxy_pack(P, bf, st, qwin);
+  if (e != cudaSuccess) return cuda_fail(e);
+  e = umma_supported(P) ? launch_score_umma(P, bf, st, K) : launch_score_simt(P, bf, st, K);
+  if (e != cudaSuccess) return cuda_fail(e);
+  if ((e = launch_mass_sum(P, bf, st)) != cudaSuccess) return cuda_fail(e);
+  return MMSHIFT_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+void mmshift_default_params(mmshift_params* p) {
+  if (!p) return;
+  std::memset(p, 0, sizeof(*p));
+  p->n_proxies = 512;
+  p->n_groups = 32;
+  p->gamma = 10.0f;
+  p->tau = 0.95f;
+  p->lambda = 1.0f;
+  p->score_mode = MMSHIFT_SCORE_VOTE;
+  p->seed = 0;
+  p->layer_id = 0;
+  p->softmax_scale = 0.0f;
+  p->rope_theta = 0.0f;
+  p->rope_pos_offset = 0;
+}
+
+mmshift_status mmshift_output_rows(const mmshift_shape* s, int64_t* rows) {
+  if (!rows) return MMSHIFT_ERR_INVALID_ARG;
+  const mmshift_status st = check_shape(s);
+  if (st != MMSHIFT_OK) return st;
+  int64_t r = 0;
+  for (int b = 0; b < s->batch; ++b)
+    r += std::min<int64_t>(s->budgets[b], (int64_t)s->cu_seqlens[b + 1] - s->cu_seqlens[b]);
+  *rows = r;
+  return MMSHIFT_OK;
+}
+
+mmshift_status mmshift_workspace_size(const mmshift_shape* s, const mmshift_params* p,
+                                      size_t* bytes) {
+  if (!bytes) return MMSHIFT_ERR_INVALID_ARG;
+  Problem P;
+  const mmshift_status st = prepare(s, p, &P);
+  if (st != MMSHIFT_OK) return st;
+  *bytes = layout_of(P).total;
+  return MMSHIFT_OK;
+}
+
+mmshift_status mmshift_build_proxies(const mmshift_shape* s, const void* Qwin,
+                                     const mmshift_params* p, void* proxies,
+                                     mmshift_stream_t stream) {
+  Problem P;
+  mmshift_status st = prepare(s, p, &P);
+  if (st != MMSHIFT_OK) return st;
+  if (!p || !Qwin || !proxies) return MMSHIFT_ERR_INVALID_ARG;
+  if (P.Np == 0) return MMSHIFT_OK;
+  Buffers bf;
+  std::memset(&bf, 0, sizeof(bf));
+  bf.proxies_out = proxies;
+  const cudaError_t e = launch_proxy_pack(P, bf, (cudaStream_t)stream, Qwin);
+  return e == cudaSuccess ? MMSHIFT_OK : cuda_fail(e);
+}
+
+mmshift_status mmshift_proxy_mass(const mmshift_shape* s, const void* K, const void* Qwin,
+                                  const void* proxies, const mmshift_params* p,
+                                  float* group_mass, float* anchor, float* mass,
+                                  void* workspace, size_t workspace_bytes,
+                                  mmshift_stream_t stream) {
+  Problem P;
+  mmshift_status st = prepare(s, p, &P);
+  if (st != MMSHIFT_OK) return st;
+  if (!p || !K || !Qwin || !anchor || (P.G && !group_mass)) return MMSHIFT_ERR_INVALID_ARG;
+  Buffers bf;
+  if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
+  bf.proxies_in = proxies;
+  if (P.G) bf.gmass = group_mass;
+  bf.anchor = anchor;
+  bf.mass = mass;
+  return run_mass(P, bf, K, Qwin, (cudaStream_t)stream);
+}
+
+mmshift_status mmshift_scores_topk(const mmshift_shape* s, const mmshift_params* p,
+                                   const float* group_mass, const float* anchor,
+                                   float* scores, int32_t* out_idx,
+                                   void* workspace, size_t workspace_bytes,
+                                   mmshift_stream_t stream) {
+  Problem P;
+  mmshift_status st = prepare(s, p, &P);
+  if (st != MMSHIFT_OK) return st;
+  if (!p || !out_idx || (P.G && !group_mass)) return MMSHIFT_ERR_INVALID_ARG;
+  if (P.mode == MMSHIFT_SCORE_VOTE && !anchor) return MMSHIFT_ERR_INVALID_ARG;
+  Buffers bf;
+  if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
+  if (P.G) bf.gmass = const_cast<float*>(group_mass);
+  if (anchor) bf.anchor = const_cast<float*>(anchor);
+  if (scores) bf.scores = scores;
+  const cudaStream_t cs = (cudaStream_t)stream;
+  cudaError_t e = cudaSuccess;
+  if (P.mode == MMSHIFT_SCORE_VOTE) e = launch_cover(P, bf, cs);
+  if (e == cudaSuccess) e = launch_topk(P, bf, cs, out_idx, false);
+  return e == cudaSuccess ? MMSHIFT_OK : cuda_fail(e);
+}
+
+mmshift_status mmshift_topk(const mmshift_shape* s, const float* scores, int32_t* out_idx,
+                            void* workspace, size_t workspace_bytes, mmshift_stream_t stream) {
+  Problem P;
+  mmshift_status st = prepare(s, nullptr, &P);
+  if (st != MMSHIFT_OK) return st;
+  if (!scores || !out_idx) return MMSHIFT_ERR_INVALID_ARG;
+  Buffers bf;
+  if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
+  bf.scores = const_cast<float*>(scores);
+  const cudaError_t e = launch_topk(P, bf, (cudaStream_t)stream, out_idx, true);
+  return e == cudaSuccess ? MMSHIFT_OK : cuda_fail(e);
+}
+
+mmshift_status mmshift_gather(const mmshift_shape* s, const void* K, const void* V,
+                              const int32_t* idx, void* out_K, void* out_V,
+                              void* workspace, size_t workspace_bytes,
+                              mmshift_stream_t stream) {
+  Problem P;
+  mmshift_status st = prepare(s, nullptr, &P);
+  if (st != MMSHIFT_OK) return st;
+  if (!K || !V || !idx || !out_K || !out_V) return MMSHIFT_ERR_INVALID_ARG;
+  Buffers bf;
+  if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
+  const cudaError_t e = launch_gather(P, bf, (cudaStream_t)stream, K, V, idx, out_K, out_V);
+  return e == cudaSuccess ? MMSHIFT_OK : cuda_fail(e);
+}
+
+mmshift_status mmshift_select(const mmshift_shape* s, const void* K, const void* V,
+                              const void* Qwin, const void* proxies_in,
+                              const mmshift_params* p, int32_t* out_idx, void* out_K,
+                              void* out_V, const mmshift_debug* dbg, void* workspace,
+                              size_t workspace_bytes, mmshift_stream_t stream) {
+  Problem P;
+  mmshift_status st = prepare(s, p, &P);
+  if (st != MMSHIFT_OK) return st;
+  if (!p || !K || !V || !Qwin || !out_idx || !out_K || !out_V) return MMSHIFT_ERR_INVALID_ARG;
+  Buffers bf;
+  if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
+  bf.proxies_in = proxies_in;
+  if (dbg) {
+    bf.proxies_out = dbg->proxies;
+    if (dbg->group_mass && P.G) bf.gmass = dbg->group_mass;
+    if (dbg->anchor) bf.anchor = dbg->anchor;
+    if (dbg->scores) bf.scores = dbg->scores;
+    bf.mass = dbg->mass;
+  }
+  const cudaStream_t cs = (cudaStream_t)stream;
+  if ((st = run_mass(P, bf, K, Qwin, cs)) != MMSHIFT_OK) return st;
+  cudaError_t e = cudaSuccess;
+  if (P.mode == MMSHIFT_SCORE_VOTE) e = launch_cover(P, bf, cs);
+  if (e == cudaSuccess) e = launch_topk(P, bf, cs, out_idx, false);
+  if (e == cudaSuccess) e = launch_gather(P, bf, cs, K, V, out_idx, out_K, out_V);
+  return e == cudaSuccess ? MMSHIFT_OK : cuda_fail(e);
+}
+
+mmshift_status mmshift_poll_status(void* workspace, mmshift_stream_t stream) {
+  if (!workspace) return MMSHIFT_ERR_INVALID_ARG;
+  cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e);
+  int word = 0;
+  if ((e = cudaMemcpy(&word, workspace, sizeof(int), cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail(e);
+  if ((e = cudaMemset(workspace, 0, sizeof(int))) != cudaSuccess) return cuda_fail(e);
+  if (word & kStatusTimeout) return MMSHIFT_ERR_TIMEOUT;
+  if (word) return MMSHIFT_ERR_DEVICE;
+  return MMSHIFT_OK;
+}
+
+const char* mmshift_status_string(mmshift_status st) {
+  switch (st) {
+    case MMSHIFT_OK: return "ok";
+    case MMSHIFT_ERR_INVALID_ARG: return "invalid argument";
+    case MMSHIFT_ERR_UNSUPPORTED: return "unsupported configuration";
+    case MMSHIFT_ERR_WORKSPACE: return "workspace missing, too small or misaligned";
+    case MMSHIFT_ERR_CUDA: return "CUDA runtime error";
+    case MMSHIFT_ERR_TIMEOUT: return "device-side wait timed out";
+    case MMSHIFT_ERR_DEVICE: return "device-side check failed";
+  }
+  return "unknown status";
+}
+
+const char* mmshift_last_cuda_error(void) { return g_cuda_error.c_str(); }
+
+}  // extern "C"

@@ -1,0 +1,132 @@
+// Internal definitions shared by the kernels and the host entry points.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "mmshift.h"
+
+namespace mmshift {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr int kChunk = 16;       // proxy rows per packing chunk (one group id)
+constexpr int kRowTile = 128;    // proxy rows are padded to a multiple of this
+
+// Status bits the kernels OR into the workspace status word.
+enum : int {
+  kStatusTimeout = 1,   // a bounded wait gave up
+  kStatusBadIndex = 2,  // gather saw an index outside [0, T_b)
+};
+
+struct ReqInfo {
+  int32_t t_len;     // T_b
+  int32_t tok_off;   // cu_seqlens[b]
+  int32_t out_off;   // sum_{b' < b} keep_{b'}
+  int32_t keep;      // min(C_b, T_b)
+  int32_t budget;    // C_b
+  int32_t word_off;  // offset of the request in a coverage bitmap row (32-bit words)
+  int32_t split_off; // first key split of the request in the softmax partials
+  int32_t nsplit;    // key splits of the request
+};
+
+// Everything a kernel needs to know about one call, passed by value.
+struct Problem {
+  int32_t B, L, Hq, Hkv, r, d, W, dtype;
+  int32_t Np, G, gs;
+  int32_t RG;          // packed rows per group: roundup(r * gs, 16)
+  int32_t n_group_rows;// G * RG
+  int32_t anchor_rows; // roundup(r, 16)
+  int32_t Prows;       // n_group_rows + anchor_rows
+  int32_t Prows_pad;   // roundup(Prows, kRowTile)
+  int32_t total_T, R, total_words, total_splits, split_len;
+  int64_t ls_kv, ls_q;
+  float scale, alpha, gamma, tau, lambda;
+  int32_t mode;
+  uint64_t seed;
+  int32_t layer_id0;
+  float rope_theta;
+  int32_t rope_off;
+  ReqInfo req[MMSHIFT_MAX_BATCH];
+};
+
+// Device buffers of one call (carved out of the caller's workspace, or the
+// caller's own debug buffers where given).
+struct Buffers {
+  int* status;
+  void* packed;       // [L][B][Hkv][Prows_pad][d] proxies, group-major rows
+  float2* part;       // [L][Hkv][total_splits][Prows_pad] (max, sum) partials
+  float* cvals;       // [L][B][Hkv][Prows_pad] log2 normaliser of each row
+  float* gmass;       // [L][Hkv][G][T]
+  float* anchor;      // [L][Hkv][T]
+  uint32_t* bits;     // [L][Hkv][G][total_words] coverage bitmaps
+  float* scores;      // [L][Hkv][T]
+  float* mass;        // [L][Hkv][T] or null
+  void* proxies_out;  // [L][B][Hq][Np][d] or null
+  const void* proxies_in; // [L][B][Hq][Np][d] or null
+};
+
+// Row p of the packed proxy block of KV head h: which group / query head /
+// proxy it holds, or that it is padding.
+struct RowKind {
+  int group;   // 0..G-1 proxy group, G = anchor, -1 = padding
+  int j;       // local query head (0..r-1)
+  int i;       // proxy index within the query head (groups only)
+};
+
+__host__ __device__ inline RowKind row_kind(const Problem& P, int p) {
+  RowKind k{-1, 0, 0};
+  if (p < P.n_group_rows) {
+    int g = p / P.RG, q = p - g * P.RG;
+    if (q < P.r * P.gs) { k.group = g; k.j = q / P.gs; k.i = g * P.gs + (q % P.gs); }
+  } else {
+    int q = p - P.n_group_rows;
+    if (q < P.r) { k.group = P.G; k.j = q; }
+  }
+  return k;
+}
+
+__host__ __device__ inline int chunk_group(const Problem& P, int chunk) {
+  int p = chunk * kChunk;
+  return p < P.n_group_rows ? p / P.RG : P.G;
+}
+
+template <typename T> __device__ __forceinline__ float to_f32(T x);
+template <> __device__ __forceinline__ float to_f32<float>(float x) { return x; }
+template <> __device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 x) {
+  return __bfloat162float(x);
+}
+template <typename T> __device__ __forceinline__ T from_f32(float x);
+template <> __device__ __forceinline__ float from_f32<float>(float x) { return x; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float x) {
+  return __float2bfloat16_rn(x);
+}
+
+__device__ __forceinline__ float fast_exp2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ void set_status(int* status, int bit) {
+  if (status) atomicOr(status, bit);
+}
+
+// Host-side launchers (one translation unit each).
+cudaError_t launch_proxy_pack(const Problem& P, const Buffers& bf, cudaStream_t st,
+                              const void* qwin);
+cudaError_t launch_score_simt(const Problem& P, const Buffers& bf, cudaStream_t st,
+                              const void* K);
+cudaError_t launch_score_umma(const Problem& P, const Buffers& bf, cudaStream_t st,
+                              const void* K);
+bool umma_supported(const Problem& P);
+cudaError_t launch_merge(const Problem& P, const Buffers& bf, cudaStream_t st);
+cudaError_t launch_cover(const Problem& P, const Buffers& bf, cudaStream_t st);
+cudaError_t launch_mass_sum(const Problem& P, const Buffers& bf, cudaStream_t st);
+cudaError_t launch_topk(const Problem& P, const Buffers& bf, cudaStream_t st,
+                        int32_t* out_idx, bool from_scores);
+cudaError_t launch_gather(const Problem& P, const Buffers& bf, cudaStream_t st,
+                          const void* K, const void* V, const int32_t* idx,
+                          void* outK, void* outV);
+
+}  // namespace mmshift

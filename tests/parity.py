@@ -1,0 +1,208 @@
+"""Helpers shared by the parity tests: run the CUDA path through the C ABI and
+the oracle on the same seeded inputs, and compare them under the tolerances
+the parity contract fixes.
+
+Tolerances (written here once, used by every GPU test):
+  * masses (group masses, anchor, summed mass): |gpu - ref| <= RTOL * |ref| + ATOL
+    with RTOL = 2e-3 (bf16 inputs, fp32 accumulation) and ATOL = 1e-9 for
+    masses that fp32 cannot resolve (the GPU flushes exp2 results below
+    2^-126 to zero);
+  * proxies: bf16 within 1 ulp, at most 1e-3 of the elements off; float32
+    within 4e-6 relative (the GPU samples in fp32, the oracle in fp64);
+  * votes: may differ only where the oracle's own decision is within the mass
+    tolerance of the tau-coverage boundary;
+  * selection: the kept set is exactly the top-(C-1) of the GPU's own scores
+    (plus T-1), and keys on which GPU and oracle disagree have oracle scores
+    within twice the largest score deviation of the cutoff;
+  * gathered K/V: bit-exact given the GPU's indices.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import paper_2607_22586_gb300 as M
+from paper_2607_22586_gb300 import synth as S
+from oracle import mmshift_oracle as O
+
+RTOL = 2e-3
+ATOL = 1e-9
+SUM_RTOL = 1e-5
+
+TORCH_DT = {S.BF16: torch.bfloat16, S.F32: torch.float32}
+ABI_DT = {S.BF16: 0, S.F32: 1}
+
+
+def f32(x: float) -> float:
+    return float(np.float32(x))
+
+
+def hyper(**kw):
+    """Hyper-parameters as the C ABI sees them (float32) for both sides."""
+    h = dict(n_proxies=512, n_groups=32, gamma=10.0, tau=0.95, lam=1.0, seed=0, layer_id=0,
+             score_mode=0, softmax_scale=0.0, rope_theta=0.0, rope_pos_offset=0)
+    h.update(kw)
+    for k in ("gamma", "tau", "lam", "softmax_scale", "rope_theta"):
+        h[k] = f32(h[k])
+    return h
+
+
+def abi_params(h):
+    return M.default_params(n_proxies=h["n_proxies"], n_groups=h["n_groups"], gamma=h["gamma"],
+                            tau=h["tau"], lam=h["lam"], seed=h["seed"], layer_id=h["layer_id"],
+                            score_mode=h["score_mode"], softmax_scale=h["softmax_scale"],
+                            rope_theta=h["rope_theta"], rope_pos_offset=h["rope_pos_offset"])
+
+
+def oracle_kw(h, dtype):
+    kw = dict(h)
+    kw["dtype"] = dtype
+    if kw["softmax_scale"] == 0.0:
+        kw["softmax_scale"] = 0.0
+    return kw
+
+
+def dev(a: np.ndarray, dtype: str) -> torch.Tensor:
+    t = torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32))
+    return t.to(TORCH_DT[dtype]).cuda().contiguous()
+
+
+def host(t: torch.Tensor) -> np.ndarray:
+    return t.float().cpu().numpy() if t.dtype != torch.int32 else t.cpu().numpy()
+
+
+def shape_of(wl: S.Workload, n_layers: int = 1, window=None):
+    w = wl.window if window is None else window
+    return M.make_shape(wl.n_q_heads, wl.n_kv_heads, wl.head_dim, w, ABI_DT[wl.dtype],
+                        wl.cu_seqlens(), wl.budgets, n_layers=n_layers,
+                        layer_stride_kv=wl.total_tokens * wl.n_kv_heads * wl.head_dim,
+                        layer_stride_q=wl.batch * w * wl.n_q_heads * wl.head_dim)
+
+
+def gpu_select(wl: S.Workload, layers, h, proxies=None):
+    """Run mmshift_select over ``layers`` (list of LayerInputs) in one call
+    with every debug output; returns numpy arrays [L, ...]."""
+    L = len(layers)
+    shape = shape_of(wl, L)
+    params = abi_params(h)
+    K = dev(np.stack([li.K for li in layers]), wl.dtype)
+    V = dev(np.stack([li.V for li in layers]), wl.dtype)
+    Q = dev(np.stack([li.Qwin for li in layers]), wl.dtype)
+    pin = dev(proxies, wl.dtype) if proxies is not None else None
+    rows = M.mmshift_output_rows(shape)
+    ws_bytes = M.mmshift_workspace_size(shape, params)
+    ws = torch.zeros(ws_bytes, dtype=torch.uint8, device="cuda")
+    hkv, hq, d, T = wl.n_kv_heads, wl.n_q_heads, wl.head_dim, wl.total_tokens
+    G = h["n_groups"]
+    out_idx = torch.full((L, rows, hkv), -7, dtype=torch.int32, device="cuda")
+    out_k = torch.empty((L, rows, hkv, d), dtype=TORCH_DT[wl.dtype], device="cuda")
+    out_v = torch.empty_like(out_k)
+    gm = torch.full((L, hkv, max(G, 1), T), -1.0, device="cuda")
+    an = torch.full((L, hkv, T), -1.0, device="cuda")
+    ms = torch.full((L, hkv, T), -1.0, device="cuda")
+    sc = torch.full((L, hkv, T), -1.0, device="cuda")
+    px = torch.empty((L, wl.batch, hq, max(h["n_proxies"], 1), d), dtype=TORCH_DT[wl.dtype], device="cuda")
+    dbg = M.make_debug(proxies=px, group_mass=gm, anchor=an, mass=ms, scores=sc)
+    st = M.mmshift_select(shape, K, V, Q, pin, params, out_idx, out_k, out_v, dbg, ws, ws_bytes)
+    M.check(st, "mmshift_select")
+    M.check(M.mmshift_poll_status(ws), "mmshift_poll_status")
+    torch.cuda.synchronize()
+    return dict(idx=host(out_idx), out_k=host(out_k), out_v=host(out_v), group_mass=host(gm),
+                anchor=host(an), mass=host(ms), scores=host(sc), proxies=host(px),
+                K=np.stack([li.K for li in layers]), V=np.stack([li.V for li in layers]))
+
+
+def oracle_layer(wl: S.Workload, li: S.LayerInputs, h, layer_id: int, proxies=None, requests=None):
+    """Oracle results for one layer: list over requests (None where skipped)."""
+    cu = wl.cu_seqlens()
+    out = []
+    kw = oracle_kw(h, wl.dtype)
+    kw["layer_id"] = layer_id
+    for b in range(wl.batch):
+        if requests is not None and b not in requests:
+            out.append(None)
+            continue
+        lo, hi = int(cu[b]), int(cu[b + 1])
+        out.append(O.select_request(li.K[lo:hi], li.V[lo:hi], li.Qwin[b], int(wl.budgets[b]), b=b,
+                                    proxies=None if proxies is None else proxies[b], **kw))
+    return out
+
+
+def mass_close(gpu: np.ndarray, ref: np.ndarray, what: str):
+    err = np.abs(gpu.astype(np.float64) - ref)
+    bound = RTOL * np.abs(ref) + ATOL
+    bad = err > bound
+    assert not bad.any(), (f"{what}: {bad.sum()} of {bad.size} outside tolerance; "
+                           f"worst rel {np.max(err / (np.abs(ref) + 1e-30)):.3g}")
+
+
+def uncertain_votes(abar: np.ndarray, tau: float) -> np.ndarray:
+    """[G, T] bool: where the oracle's coverage decision is within tolerance."""
+    G, T = abar.shape
+    unc = np.zeros((G, T), dtype=bool)
+    for g in range(G):
+        order = np.lexsort((np.arange(T), -abar[g]))
+        csum = np.cumsum(abar[g][order])
+        total = csum[-1]
+        target = tau * total
+        eps = SUM_RTOL * total + ATOL
+        k = int(np.argmax(csum >= target))
+        theta = abar[g][order[k]]
+        before = np.concatenate([[0.0], csum[:-1]])
+        near_sum = (before <= target + eps) & (csum >= target - eps)
+        near_val = np.abs(abar[g][order] - theta) <= RTOL * theta + ATOL
+        unc[g, order] = near_sum | near_val
+    return unc
+
+
+def check_request(gpu, ref, h, lo, hi, layer, what=""):
+    """Compare one request of one layer: masses, anchor, votes, scores, selection, gather."""
+    G, tau, lam, mode = h["n_groups"], h["tau"], h["lam"], h["score_mode"]
+    hkv = ref["anchor"].shape[0]
+    T = hi - lo
+    if G:
+        mass_close(gpu["group_mass"][layer][:, :G, lo:hi], ref["group_mass"], what + " group_mass")
+    mass_close(gpu["anchor"][layer][:, lo:hi], ref["anchor"], what + " anchor")
+    mass_close(gpu["mass"][layer][:, lo:hi], ref["mass"], what + " mass")
+    s_gpu = gpu["scores"][layer][:, lo:hi].astype(np.float64)
+    s_ref = ref["scores"]
+    if mode == O.SCORE_VOTE and G:
+        for hh in range(hkv):
+            unc = uncertain_votes(ref["group_mass"][hh], tau)
+            v_ref = O.votes(O.cover_sets(ref["group_mass"][hh], tau))
+            anc_gpu = gpu["anchor"][layer][hh, lo:hi].astype(np.float64)
+            v_gpu = np.rint(s_gpu[hh] - np.float32(lam) * anc_gpu)
+            dv = np.abs(v_gpu - v_ref)
+            assert np.all(dv <= unc.sum(axis=0)), f"{what} head {hh}: vote mismatch outside band"
+    dev_max = np.max(np.abs(s_gpu - s_ref)) if T else 0.0
+    keep_rows = ref["idx"].shape[0]
+    idx_gpu = gpu["idx"][layer]
+    for hh in range(hkv):
+        got = idx_gpu[:, hh]
+        assert got.shape[0] == keep_rows
+        assert np.all(np.diff(got) > 0) and got[-1] == T - 1 and got[0] >= 0, f"{what}: malformed idx"
+        # self-consistency: exactly the top-(C-1) of the GPU's own scores
+        if keep_rows < T:
+            cand = np.arange(T - 1)
+            order = np.lexsort((cand, -gpu["scores"][layer][hh, lo:hi - 1].astype(np.float64)))
+            expect = np.sort(np.concatenate([order[:keep_rows - 1], [T - 1]]))
+            np.testing.assert_array_equal(got, expect, err_msg=f"{what}: not the top-k of own scores")
+            diff = set(got.tolist()) ^ set(ref["idx"][:, hh].tolist())
+            if diff:
+                srt = np.sort(s_ref[hh][:T - 1])[::-1]
+                cut = srt[keep_rows - 2]
+                band = 2.0 * dev_max + 1e-6
+                far = [t for t in diff if abs(s_ref[hh][t] - cut) > band]
+                assert not far, f"{what} head {hh}: {len(far)} selection mismatches outside the band"
+        else:
+            np.testing.assert_array_equal(got, np.arange(T))
+    return dev_max
+
+
+def check_gather(gpu, wl, layer, lo_tok, out_lo, keep, T, hkv):
+    idx = gpu["idx"][layer][out_lo:out_lo + keep]
+    h = np.arange(hkv)[None, :]
+    kref = gpu["K"][layer][lo_tok + idx, h]
+    vref = gpu["V"][layer][lo_tok + idx, h]
+    np.testing.assert_array_equal(gpu["out_k"][layer][out_lo:out_lo + keep], kref)
+    np.testing.assert_array_equal(gpu["out_v"][layer][out_lo:out_lo + keep], vref)

@@ -1,0 +1,95 @@
+"""Host-side checks of the C ABI that need no GPU: the library builds and
+loads, exports every entry point declared in include/mmshift.h, and rejects
+bad arguments before touching the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2607_22586_gb300 as M
+from paper_2607_22586_gb300 import _lib as L
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_entry_points():
+    with open(os.path.join(ROOT, "include", "mmshift.h")) as f:
+        text = f.read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(mmshift_[a-z_0-9]+)\s*\(", text)))
+
+
+def test_library_exports_every_declared_symbol():
+    lib = M.load_library()
+    names = declared_entry_points()
+    assert len(names) >= 12
+    for n in names:
+        assert hasattr(lib, n), n
+    assert sorted(L.EXPORTED) == names
+
+
+def test_default_params_are_the_papers():
+    p = M.default_params()
+    assert (p.n_proxies, p.n_groups) == (512, 32)
+    assert p.gamma == 10.0 and p.lambda_ == 1.0
+    assert abs(p.tau - 0.95) < 1e-7
+    assert p.score_mode == L.MMSHIFT_SCORE_VOTE
+
+
+def _shape(**kw):
+    base = dict(n_q_heads=8, n_kv_heads=2, head_dim=128, window=8, dtype=0,
+                cu_seqlens=[0, 100, 250], budgets=[16, 300])
+    base.update(kw)
+    return M.make_shape(**base)
+
+
+def test_output_rows_and_workspace():
+    s = _shape()
+    assert M.mmshift_output_rows(s) == 16 + 150
+    n = M.mmshift_workspace_size(s, M.default_params())
+    assert n > 0 and n % 256 == 0
+
+
+@pytest.mark.parametrize("bad,code", [
+    (dict(n_q_heads=7), L.MMSHIFT_ERR_INVALID_ARG),      # Hq not a multiple of Hkv
+    (dict(window=1), L.MMSHIFT_ERR_INVALID_ARG),         # std needs W >= 2
+    (dict(head_dim=96), L.MMSHIFT_ERR_UNSUPPORTED),
+    (dict(dtype=5), L.MMSHIFT_ERR_UNSUPPORTED),
+    (dict(cu_seqlens=[0, 100, 100]), L.MMSHIFT_ERR_INVALID_ARG),   # empty request
+    (dict(cu_seqlens=[1, 100, 200]), L.MMSHIFT_ERR_INVALID_ARG),
+    (dict(budgets=[16, 0]), L.MMSHIFT_ERR_INVALID_ARG),
+])
+def test_bad_shapes_rejected(bad, code):
+    s = _shape(**bad)
+    with pytest.raises(L.MMShiftError) as ei:
+        M.mmshift_workspace_size(s, M.default_params())
+    assert ei.value.code == code
+
+
+@pytest.mark.parametrize("bad", [
+    dict(n_proxies=500), dict(n_groups=0), dict(gamma=0.0), dict(tau=0.0), dict(tau=1.5),
+    dict(lam=-1.0), dict(score_mode=7), dict(layer_id=-1), dict(softmax_scale=-1.0),
+])
+def test_bad_params_rejected(bad):
+    p = M.default_params(**bad)
+    with pytest.raises(L.MMShiftError) as ei:
+        M.mmshift_workspace_size(_shape(), p)
+    assert ei.value.code == L.MMSHIFT_ERR_INVALID_ARG
+
+
+def test_null_and_workspace_errors_return_before_any_launch():
+    s = _shape()
+    p = M.default_params()
+    n = M.mmshift_workspace_size(s, p)
+    fake = 1 << 40  # never dereferenced: validation fails first
+    assert M.mmshift_select(s, None, fake, fake, None, p, fake, fake, fake, None, fake, n) == \
+        L.MMSHIFT_ERR_INVALID_ARG
+    assert M.mmshift_select(s, fake, fake, fake, None, p, fake, fake, fake, None, fake, n - 256) == \
+        L.MMSHIFT_ERR_WORKSPACE
+    assert M.mmshift_select(s, fake, fake, fake, None, p, fake, fake, fake, None, fake + 8, n) == \
+        L.MMSHIFT_ERR_WORKSPACE
+    assert M.mmshift_topk(s, None, fake, fake, n) == L.MMSHIFT_ERR_INVALID_ARG
+    assert M.mmshift_gather(s, fake, fake, None, fake, fake, fake, n) == L.MMSHIFT_ERR_INVALID_ARG
+    lib = M.load_library()
+    assert lib.mmshift_status_string(L.MMSHIFT_ERR_TIMEOUT) == b"device-side wait timed out"

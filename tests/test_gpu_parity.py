@@ -1,0 +1,220 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle on the
+same seeded inputs, element by element, with the tolerances of tests/parity.py.
+"""
+import numpy as np
+import pytest
+import torch
+
+import paper_2607_22586_gb300 as M
+from paper_2607_22586_gb300 import synth as S
+from oracle import mmshift_oracle as O
+from tests import parity as PT
+
+pytestmark = pytest.mark.gpu
+
+TINY = S.WORKLOADS["tiny-f32"]
+QWEN1 = S.WORKLOADS["qwen7b-1layer"]
+# ragged, 72B-head-shaped, small enough for the oracle: several key tiles and tails
+RAGGED = S.WORKLOADS["72b-80l-ragged"].replace(
+    name="ragged-small", n_layers=1, seq_lens=(300, 1000, 77, 2), n_visual=(285, 950, 73, 0),
+    budgets=(64, 2000, 16, 1), n_centres=32)
+
+
+def _requests(wl):
+    cu = wl.cu_seqlens()
+    outs = np.concatenate([[0], np.cumsum(np.minimum(wl.budgets, wl.seq_lens))])
+    return [(b, int(cu[b]), int(cu[b + 1]), int(outs[b])) for b in range(wl.batch)]
+
+
+def _check_all(wl, gpu, refs, h, layer=0, what=""):
+    for b, lo, hi, olo in _requests(wl):
+        if refs[b] is None:
+            continue
+        PT.check_request(gpu, refs[b], h, lo, hi, layer, f"{what} req {b}")
+        PT.check_gather(gpu, wl, layer, lo, olo, min(wl.budgets[b], hi - lo), hi - lo, wl.n_kv_heads)
+
+
+# ---------------------------------------------------------------------------
+# step 1: proxies
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("name,rope", [("tiny-f32", 0.0), ("qwen7b-1layer", 0.0),
+                                       ("qwen7b-1layer", 1e6), ("ragged-small", 0.0)])
+def test_proxies_match_oracle(name, rope):
+    wl = RAGGED if name == "ragged-small" else S.WORKLOADS[name]
+    li = S.make_layer(wl, 0)
+    h = PT.hyper(seed=1234, layer_id=5, rope_theta=rope, rope_pos_offset=3)
+    shape = PT.shape_of(wl)
+    Q = PT.dev(li.Qwin, wl.dtype)
+    out = torch.empty((1, wl.batch, wl.n_q_heads, h["n_proxies"], wl.head_dim),
+                      dtype=PT.TORCH_DT[wl.dtype], device="cuda")
+    M.check(M.mmshift_build_proxies(shape, Q, PT.abi_params(h), out), "build_proxies")
+    got = PT.host(out)[0].astype(np.float64)
+    for b in range(wl.batch):
+        z = O.proxy_normals(h["seed"], h["layer_id"], b, wl.n_q_heads, h["n_proxies"], wl.head_dim)
+        ref = O.build_proxies(li.Qwin[b], z, h["gamma"], wl.seq_lens[b], wl.dtype, rope,
+                              h["rope_pos_offset"])
+        if wl.dtype == S.BF16:
+            _, e = np.frexp(np.maximum(np.abs(ref), np.abs(got[b])))
+            ulp = np.ldexp(1.0, e - 8)
+            diff = np.abs(got[b] - ref)
+            assert np.all(diff <= ulp * 1.0001), "bf16 proxies off by more than one ulp"
+            frac = np.mean(diff > 0)
+            assert frac <= 1e-3, f"{frac:.2e} of proxies differ by one ulp"
+        else:
+            np.testing.assert_allclose(got[b], ref, rtol=4e-6, atol=1e-6)
+
+
+# ---------------------------------------------------------------------------
+# steps 2-6 with identical (given) proxies
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("name", ["tiny-f32", "qwen7b-1layer", "ragged-small"])
+@pytest.mark.parametrize("mode", [O.SCORE_VOTE, O.SCORE_MASS])
+def test_select_given_proxies(name, mode):
+    wl = RAGGED if name == "ragged-small" else S.WORKLOADS[name]
+    li = S.make_layer(wl, 0)
+    h = PT.hyper(score_mode=mode)
+    prox = S.make_proxies(wl, h["n_proxies"], 0)
+    gpu = PT.gpu_select(wl, [li], h, proxies=prox[None])
+    refs = PT.oracle_layer(wl, li, h, 0, proxies=prox)
+    _check_all(wl, gpu, refs, h, what=name)
+
+
+@pytest.mark.parametrize("kw", [dict(n_proxies=64, n_groups=4), dict(n_proxies=128, n_groups=32),
+                                dict(tau=1.0), dict(tau=0.5, lam=0.0), dict(n_proxies=0, n_groups=0),
+                                dict(n_proxies=32, n_groups=2, softmax_scale=0.05)])
+def test_select_hyperparameters(kw):
+    wl = QWEN1.replace(seq_lens=(1500,), n_visual=(1400,), budgets=(200,))
+    li = S.make_layer(wl, 3)
+    h = PT.hyper(**kw)
+    prox = S.make_proxies(wl, max(h["n_proxies"], 1), 3)[:, :, :h["n_proxies"]]
+    pin = prox if h["n_proxies"] else None
+    gpu = PT.gpu_select(wl, [li], h, proxies=None if pin is None else pin[None])
+    refs = PT.oracle_layer(wl, li, h, 0, proxies=pin)
+    _check_all(wl, gpu, refs, h, what=str(kw))
+
+
+def test_multi_layer_call_matches_single_layer_calls():
+    wl = RAGGED.replace(seq_lens=(200, 333), n_visual=(190, 300), budgets=(50, 64))
+    lis = [S.make_layer(wl, l) for l in range(3)]
+    h = PT.hyper(n_proxies=64, n_groups=4, seed=9, layer_id=2)
+    multi = PT.gpu_select(wl, lis, h)
+    for l in range(3):
+        single = PT.gpu_select(wl, [lis[l]], dict(h, layer_id=2 + l))
+        for key in ("idx", "out_k", "group_mass", "anchor", "scores", "proxies"):
+            np.testing.assert_array_equal(multi[key][l], single[key][0], err_msg=key)
+
+
+# ---------------------------------------------------------------------------
+# end to end with the sampled proxies
+# ---------------------------------------------------------------------------
+def test_end_to_end_sampled_f32():
+    wl = TINY
+    li = S.make_layer(wl, 0)
+    h = PT.hyper(seed=3)
+    gpu = PT.gpu_select(wl, [li], h)
+    refs = PT.oracle_layer(wl, li, h, 0)
+    _check_all(wl, gpu, refs, h, what="tiny sampled")
+
+
+def test_end_to_end_sampled_bf16_agreement():
+    """bf16 proxies may differ from the oracle's by one ulp in a few elements
+    (fp32 vs fp64 sampling), which moves single logits; the selection must
+    still agree on almost every key."""
+    wl = QWEN1
+    li = S.make_layer(wl, 0)
+    h = PT.hyper(seed=3)
+    gpu = PT.gpu_select(wl, [li], h)
+    ref = PT.oracle_layer(wl, li, h, 0)[0]
+    err = np.abs(gpu["group_mass"][0][:, :, :].astype(np.float64) - ref["group_mass"])
+    bad = err > PT.RTOL * np.abs(ref["group_mass"]) + PT.ATOL
+    assert bad.mean() < 1e-3, f"{bad.mean():.2e} of group masses outside tolerance"
+    for hh in range(wl.n_kv_heads):
+        a, b = set(gpu["idx"][0][:, hh].tolist()), set(ref["idx"][:, hh].tolist())
+        assert len(a & b) >= 0.98 * len(b), f"head {hh}: overlap {len(a & b)}/{len(b)}"
+
+
+# ---------------------------------------------------------------------------
+# selection steps alone, on generated masses / scores (exact)
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("tau", [0.95, 0.5, 1.0])
+def test_scores_topk_exact_on_generated_masses(tau):
+    wl = RAGGED.replace(seq_lens=(700, 2500, 40), n_visual=(600, 2400, 30), budgets=(100, 300, 8))
+    h = PT.hyper(n_proxies=64, n_groups=8, tau=tau)
+    T, hkv, G = wl.total_tokens, wl.n_kv_heads, h["n_groups"]
+    gm = S.make_group_masses(hkv, G, T, 112.0, seed=5)
+    # masses per request must be each request's own distribution
+    anchor = S.make_scores(hkv, T, 0, seed=6) * np.float32(0.5)
+    shape = PT.shape_of(wl)
+    params = PT.abi_params(h)
+    ws_bytes = M.mmshift_workspace_size(shape, params)
+    ws = torch.zeros(ws_bytes, dtype=torch.uint8, device="cuda")
+    rows = M.mmshift_output_rows(shape)
+    idx = torch.full((1, rows, hkv), -1, dtype=torch.int32, device="cuda")
+    sc = torch.empty((1, hkv, T), device="cuda")
+    st = M.mmshift_scores_topk(shape, params, torch.from_numpy(gm).cuda(),
+                               torch.from_numpy(anchor).cuda(), sc, idx, ws, ws_bytes)
+    M.check(st, "scores_topk")
+    torch.cuda.synchronize()
+    sc, idx = PT.host(sc)[0], PT.host(idx)[0]
+    for b, lo, hi, olo in _requests(wl):
+        keep = min(wl.budgets[b], hi - lo)
+        for hh in range(hkv):
+            v = O.votes(O.cover_sets(gm[hh, :, lo:hi].astype(np.float64), tau))
+            s_exp = (v.astype(np.float32) + np.float32(h["lam"]) * anchor[hh, lo:hi]).astype(np.float32)
+            np.testing.assert_array_equal(sc[hh, lo:hi], s_exp)
+            np.testing.assert_array_equal(idx[olo:olo + keep, hh],
+                                          O.select_topk(s_exp.astype(np.float64), wl.budgets[b]))
+
+
+@pytest.mark.parametrize("lens,budgets", [((5000,), (700,)), ((1, 2, 3, 64, 65), (1, 1, 2, 10, 64)),
+                                          ((60000,), (4096,)), ((33, 4097), (32, 4097))])
+def test_topk_exact_on_generated_scores(lens, budgets):
+    wl = RAGGED.replace(seq_lens=lens, n_visual=tuple(0 for _ in lens), budgets=budgets)
+    T, hkv = wl.total_tokens, wl.n_kv_heads
+    s = S.make_scores(hkv, T, 32, seed=len(lens))
+    shape = PT.shape_of(wl)
+    ws_bytes = M.mmshift_workspace_size(shape, None)
+    ws = torch.zeros(ws_bytes, dtype=torch.uint8, device="cuda")
+    rows = M.mmshift_output_rows(shape)
+    idx = torch.full((1, rows, hkv), -1, dtype=torch.int32, device="cuda")
+    M.check(M.mmshift_topk(shape, torch.from_numpy(s).cuda(), idx, ws, ws_bytes), "topk")
+    torch.cuda.synchronize()
+    idx = PT.host(idx)[0]
+    for b, lo, hi, olo in _requests(wl):
+        keep = min(budgets[b], hi - lo)
+        for hh in range(hkv):
+            np.testing.assert_array_equal(idx[olo:olo + keep, hh],
+                                          O.select_topk(s[hh, lo:hi].astype(np.float64), budgets[b]))
+
+
+def test_gather_bit_exact_and_bad_index_reported():
+    wl = RAGGED
+    li = S.make_layer(wl, 1)
+    shape = PT.shape_of(wl)
+    rows = M.mmshift_output_rows(shape)
+    rng = np.random.default_rng(0)
+    idx = np.zeros((rows, wl.n_kv_heads), dtype=np.int32)
+    for b, lo, hi, olo in _requests(wl):
+        keep = min(wl.budgets[b], hi - lo)
+        idx[olo:olo + keep] = rng.integers(0, hi - lo, size=(keep, wl.n_kv_heads))
+    K, V = PT.dev(li.K, wl.dtype), PT.dev(li.V, wl.dtype)
+    ok, ov = (torch.empty((1, rows, wl.n_kv_heads, wl.head_dim), dtype=torch.bfloat16, device="cuda")
+              for _ in range(2))
+    ws_bytes = M.mmshift_workspace_size(shape, None)
+    ws = torch.zeros(ws_bytes, dtype=torch.uint8, device="cuda")
+    M.check(M.mmshift_gather(shape, K, V, torch.from_numpy(idx).cuda(), ok, ov, ws, ws_bytes), "gather")
+    assert M.mmshift_poll_status(ws) == 0
+    ok, ov = PT.host(ok)[0], PT.host(ov)[0]
+    hh = np.arange(wl.n_kv_heads)[None]
+    for b, lo, hi, olo in _requests(wl):
+        keep = min(wl.budgets[b], hi - lo)
+        np.testing.assert_array_equal(ok[olo:olo + keep], li.K[lo + idx[olo:olo + keep], hh])
+        np.testing.assert_array_equal(ov[olo:olo + keep], li.V[lo + idx[olo:olo + keep], hh])
+    # an out-of-range index: row zero-filled, status reported, context intact
+    idx[0, 0] = 10 ** 6
+    M.check(M.mmshift_gather(shape, K, V, torch.from_numpy(idx).cuda(), ok_t := torch.empty(
+        (1, rows, wl.n_kv_heads, wl.head_dim), dtype=torch.bfloat16, device="cuda"),
+        torch.empty_like(ok_t), ws, ws_bytes), "gather")
+    assert M.mmshift_poll_status(ws) == M._lib.MMSHIFT_ERR_DEVICE
+    assert torch.all(ok_t[0, 0, 0] == 0)
+    assert M.mmshift_poll_status(ws) == 0
