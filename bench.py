@@ -1,0 +1,417 @@
+#!/usr/bin/env python3
+"""Benchmark: prefill-only KV selection throughput on GB300.
+
+One step = one mmshift_select call over every layer of the workload (proxies,
+two-pass proxy softmax with group-mass aggregation, coverage vote, budgeted
+top-k, gather), inputs resident in HBM. Default workload: the 28-layer
+Qwen2.5-VL-7B-shaped long-context stack (T = 32768 = 4 images x 8064 visual +
+512 text tokens, Hq/Hkv = 28/4, d = 128, bf16, window 32, budget 2048) with the
+paper's hyper-parameters (N = 512 proxies, G = 32, gamma = 10, tau = 0.95,
+lambda = 1).
+
+Metric: prompt tokens selected per second per layer (sum_b T_b * L / step
+time), whole job over all ranks; plus the fraction of the HBM roofline the
+step's algorithmic bytes (K read once + K/V gathered, read and written) reach.
+
+--impl reference times the CPU oracle on the host cores instead (a bounded
+sample of the same workload per step).
+
+Multi-GPU (torchrun): every rank runs its own replica of the workload (units
+are independent: no data-path collective); value sums all ranks' tokens over
+the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import multiprocessing as mp
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2607_22586_gb300 import synth as S  # noqa: E402
+
+METRIC = "prompt tokens selected/sec per layer + % of GB300 HBM roofline (bytes read/time)"
+UNIT = "tokens/s/layer"
+SM_COUNT = 152
+FP32_LANES_PER_SM = 128
+
+
+def _gen_one(args):
+    wl, layer = args
+    li = S.make_layer(wl, layer)
+    return li.native(wl.dtype)
+
+
+def gen_workload(wl, rank_seed: int, procs: int):
+    """All layers of wl as stacked native arrays (K, V, Qwin), seeded."""
+    wl = wl.replace(seed=wl.seed + rank_seed)
+    jobs = [(wl, l) for l in range(wl.n_layers)]
+    if procs > 1 and wl.n_layers > 1:
+        with mp.get_context("spawn").Pool(procs) as pool:
+            parts = pool.map(_gen_one, jobs)
+    else:
+        parts = [_gen_one(j) for j in jobs]
+    return tuple(np.stack([p[i] for p in parts]) for i in range(3))
+
+
+def read_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                "sm_max_mhz": 2070.0}, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = max(mx, float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        load = [x for x in sm if x > 0.5 * max(sm)] or sm
+        return {"sm_mhz": statistics.median(load), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def oracle_sample_rate(wl, K, V, Q, hyper, budget_s: float):
+    """Run the oracle on (layer, KV head) units of the workload until about
+    ``budget_s`` seconds of CPU work; return (tokens/s/layer, description)."""
+    from oracle import mmshift_oracle as O
+    r = wl.n_q_heads // wl.n_kv_heads
+    cu = wl.cu_seqlens()
+    done, spent, units = 0.0, 0.0, 0
+    to_f = (lambda a: S.bf16_bits_to_f32(a)) if wl.dtype == S.BF16 else (lambda a: a)
+    for layer in range(wl.n_layers):
+        for h in range(wl.n_kv_heads):
+            for b in range(wl.batch):
+                lo, hi = int(cu[b]), int(cu[b + 1])
+                k = to_f(K[layer, lo:hi, h:h + 1])
+                v = to_f(V[layer, lo:hi, h:h + 1])
+                q = to_f(Q[layer, b, :, h * r:(h + 1) * r])
+                t0 = time.perf_counter()
+                O.select_request(k, v, q, int(wl.budgets[b]), b=b, layer_id=layer, dtype=wl.dtype,
+                                 **hyper)
+                spent += time.perf_counter() - t0
+                done += (hi - lo) / wl.n_kv_heads     # one head = 1/Hkv of a layer
+                units += 1
+                if spent >= budget_s:
+                    return done / spent, f"{units} (layer, KV head, request) units of the workload"
+    return done / spent, f"{units} (layer, KV head, request) units (whole workload)"
+
+
+def blas_threads() -> int:
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads", 1) for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    return int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+
+
+def hyper_for(args, wl):
+    if args.proxies == "few":
+        n_p = wl.window
+        return dict(n_proxies=n_p, n_groups=max(1, n_p // 16), gamma=10.0, tau=float(np.float32(0.95)),
+                    lam=1.0, seed=0)
+    return dict(n_proxies=512, n_groups=32, gamma=10.0, tau=float(np.float32(0.95)), lam=1.0, seed=0)
+
+
+def algorithmic(wl, hyper):
+    """Per step: HBM bytes (K read once + K/V gathered read+write) and the
+    logits of one softmax pass (2 d flops per (proxy row, key))."""
+    esz = 2 if wl.dtype == S.BF16 else 4
+    L, hkv, d = wl.n_layers, wl.n_kv_heads, wl.head_dim
+    T = wl.total_tokens
+    keep = sum(min(c, t) for c, t in zip(wl.budgets, wl.seq_lens))
+    k_read = L * T * hkv * d * esz
+    gather = 4 * L * keep * hkv * d * esz
+    r = wl.n_q_heads // hkv
+    rows = hyper["n_proxies"] * r + r       # proxies of the r query heads + anchor rows
+    pass_flops = 2.0 * d * rows * T * hkv * L
+    return k_read + gather, k_read, pass_flops
+
+
+def run_reference(args, wl):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    hyper = hyper_for(args, wl)
+    # one layer of the workload is enough to sample from
+    wl1 = wl.replace(n_layers=1)
+    K, V, Q = gen_workload(wl1, 0, 1)
+    for _ in range(args.warmup):
+        oracle_sample_rate(wl1, K, V, Q, hyper, budget_s=0.0)
+    rates, t0 = [], time.perf_counter()
+    for _ in range(args.steps):
+        rate, sample = oracle_sample_rate(wl1, K, V, Q, hyper, budget_s=args.ref_seconds)
+        rates.append(rate)
+    wall = time.perf_counter() - t0
+    value = statistics.mean(rates)
+    cores = blas_threads()
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * wall / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded, MLLM-shaped)",
+        "config": {"workload": wl.name, "proxies": args.proxies, **{k: hyper[k] for k in ("n_proxies", "n_groups")}},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": f"per step: {sample}; numpy float64 (BLAS matmul threads={cores}, "
+                                   f"elementwise single-threaded)"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_gpu(args, wl):
+    import torch
+    import paper_2607_22586_gb300 as M
+    from paper_2607_22586_gb300 import _lib as LB
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.device("cuda", torch.cuda.current_device())
+    hyper = hyper_for(args, wl)
+    peaks, peak_src = read_peaks()
+
+    # inputs: seeded on the host (replica r of the workload on rank r)
+    t0 = time.perf_counter()
+    Kh, Vh, Qh = gen_workload(wl, rank, args.gen_procs)
+    gen_s = time.perf_counter() - t0
+    tdt = torch.bfloat16 if wl.dtype == S.BF16 else torch.float32
+    as_t = (lambda a: torch.from_numpy(a.view(np.int16)).view(torch.bfloat16)) if wl.dtype == S.BF16 \
+        else (lambda a: torch.from_numpy(a))
+    K_pin, V_pin, Q_pin = (as_t(a).pin_memory() for a in (Kh, Vh, Qh))
+    K, V, Q = (t.to(dev) for t in (K_pin, V_pin, Q_pin))
+
+    L = wl.n_layers
+    T = wl.total_tokens
+    shape = M.make_shape(wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.window,
+                         0 if wl.dtype == S.BF16 else 1, wl.cu_seqlens(), wl.budgets, n_layers=L,
+                         layer_stride_kv=T * wl.n_kv_heads * wl.head_dim,
+                         layer_stride_q=wl.batch * wl.window * wl.n_q_heads * wl.head_dim)
+    params = M.default_params(n_proxies=hyper["n_proxies"], n_groups=hyper["n_groups"],
+                              gamma=hyper["gamma"], tau=hyper["tau"], lam=hyper["lam"], seed=hyper["seed"])
+    rows = M.mmshift_output_rows(shape)
+    ws_bytes = M.mmshift_workspace_size(shape, params)
+    ws = torch.zeros(ws_bytes, dtype=torch.uint8, device=dev)
+    out_idx = torch.empty((L, rows, wl.n_kv_heads), dtype=torch.int32, device=dev)
+    out_k = torch.empty((L, rows, wl.n_kv_heads, wl.head_dim), dtype=tdt, device=dev)
+    out_v = torch.empty_like(out_k)
+    stream = torch.cuda.current_stream(dev)
+    nst = LB.MMSHIFT_N_STAGES + 1
+
+    def step(dbg=None):
+        M.check(M.mmshift_select(shape, K, V, Q, None, params, out_idx, out_k, out_v, dbg, ws,
+                                 ws_bytes, stream), "mmshift_select")
+
+    for _ in range(args.warmup):
+        step()
+    M.check(M.mmshift_poll_status(ws, stream), "warm-up status")
+
+    # device-timed steps: inputs resident in HBM and larger than L2
+    stage_ev = [[torch.cuda.Event(enable_timing=True) for _ in range(nst)] for _ in range(args.steps)]
+    for evs in stage_ev:          # torch creates the CUDA event on first record
+        for ev in evs:
+            ev.record(stream)
+    dbgs = [M.make_debug(stage_events=ev) for ev in stage_ev]
+    clocks = ClockSampler(torch.cuda.current_device())
+    clocks.start()
+    time.sleep(0.3)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for k in range(args.steps):
+        step(dbgs[k])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    clk = clocks.stop()
+    M.check(M.mmshift_poll_status(ws, stream), "timed status")
+    ms = t_start.elapsed_time(t_end) / args.steps
+    if dist:
+        tt = torch.tensor([ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    stage_ms = {name: statistics.mean(ev[i].elapsed_time(ev[i + 1]) for ev in stage_ev)
+                for i, name in enumerate(LB.STAGES)}
+    launches = dbgs[0].launches * args.steps
+
+    # end to end through the same C ABI call: host buffers in, results out
+    idx_h = torch.empty(out_idx.shape, dtype=out_idx.dtype, pin_memory=True)
+    ok_h = torch.empty(out_k.shape, dtype=out_k.dtype, pin_memory=True)
+    ov_h = torch.empty_like(ok_h, pin_memory=True)
+    e_steps = max(1, args.steps)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(e_steps):
+        K.copy_(K_pin, non_blocking=True)
+        V.copy_(V_pin, non_blocking=True)
+        Q.copy_(Q_pin, non_blocking=True)
+        step()
+        idx_h.copy_(out_idx, non_blocking=True)
+        ok_h.copy_(out_k, non_blocking=True)
+        ov_h.copy_(out_v, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e_ms = e0.elapsed_time(e1) / e_steps
+    if dist:
+        tt = torch.tensor([e_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e_ms = float(tt.item())
+    h2d = sum(t.numel() * t.element_size() for t in (K_pin, V_pin, Q_pin))
+    d2h = sum(t.numel() * t.element_size() for t in (idx_h, ok_h, ov_h))
+
+    bytes_step, k_read, pass_flops = algorithmic(wl, hyper)
+    tokens_layer = T * L * world
+    value = tokens_layer / (ms * 1e-3)
+    hbm_frac = bytes_step / (ms * 1e-3) / (peaks["hbm_gbs"] * 1e9)
+
+    # dominant stage and its roofline
+    dom = max(("softmax_pass", "mass_pass"), key=lambda s: stage_ms[s])
+    dom_ms = stage_ms[dom]
+    umma = dbgs[0].score_path == 1
+    if umma:
+        achieved = pass_flops / (dom_ms * 1e-3) / 1e12
+        peak = float(peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]))
+        roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": achieved / peak, "traffic": None, "kernel": dom,
+                "peak_kind": f"bf16 dense, sustained ({peak_src})"}
+    else:
+        achieved = pass_flops / (dom_ms * 1e-3) / 1e12
+        mhz = float(peaks.get("sm_max_mhz", 2070.0))
+        peak = SM_COUNT * FP32_LANES_PER_SM * 2 * mhz * 1e6 / 1e12
+        roof = {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": achieved / peak, "traffic": None, "kernel": dom,
+                "peak_kind": f"fp32 FMA: {SM_COUNT} SMs x {FP32_LANES_PER_SM} lanes x 2 flop x {mhz:.0f} MHz"}
+
+    cpu = None
+    if rank == 0 and args.cpu_seconds > 0:
+        rate, sample = oracle_sample_rate(wl, Kh, Vh, Qh, hyper, budget_s=args.cpu_seconds)
+        cores = blas_threads()
+        cpu = {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
+               "sample": f"{sample}, about {args.cpu_seconds:.0f} s; numpy float64 "
+                         f"(BLAS matmul threads={cores}, elementwise single-threaded)"}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16" if wl.dtype == S.BF16 else "f32",
+        "data": "synthetic (seeded, MLLM-shaped; stands in for the paper's benchmarks)",
+        "config": {"workload": wl.name, "layers": L, "batch": wl.batch, "prompt_tokens": T,
+                   "q_heads": wl.n_q_heads, "kv_heads": wl.n_kv_heads, "head_dim": wl.head_dim,
+                   "window": wl.window, "budgets": list(wl.budgets), "proxies": args.proxies,
+                   "n_proxies": hyper["n_proxies"], "n_groups": hyper["n_groups"],
+                   "gamma": hyper["gamma"], "tau": hyper["tau"], "lambda": hyper["lam"],
+                   "l2": "inputs (K+V %.2f GB) larger than L2; no flush" % (2 * k_read / 1e9),
+                   "parallelism": f"replicas x{world}"},
+        "hbm_roofline_frac": hbm_frac,
+        "hbm_bytes_per_step": bytes_step,
+        "stage_ms": stage_ms,
+        "roofline": roof,
+        "cpu_baseline": cpu,
+        "e2e": {"value": tokens_layer / (e_ms * 1e-3), "unit": UNIT, "ms_per_step": e_ms,
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "clocks": clk,
+        "gpu_launches": launches,
+        "input_gen_s": gen_s,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="qwen7b-28l-32k", choices=sorted(S.WORKLOADS))
+    ap.add_argument("--proxies", choices=["paper", "few"], default="paper",
+                    help="paper: N=512, G=32 (Section 4.1); few: N=W, G=W/16")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0,
+                    help="CPU oracle sample budget for cpu_baseline (0 disables)")
+    ap.add_argument("--ref-seconds", type=float, default=8.0,
+                    help="per-step oracle sample budget of --impl reference")
+    ap.add_argument("--gen-procs", type=int, default=min(8, os.cpu_count() or 1))
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    wl = S.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        return run_reference(args, wl)
+    return run_gpu(args, wl)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -114,7 +114,20 @@ typedef struct {
   float* anchor;     /* [L, Hkv, T] last-query attention, mean over the GQA heads */
   float* mass;       /* [L, Hkv, T] sum_g group_mass */
   float* scores;     /* [L, Hkv, T] S_t used by the top-k */
+  /* Stage timing: if n_stage_events >= MMSHIFT_N_STAGES + 1, stage_events
+   * holds caller-created cudaEvent_t handles and event i is recorded on
+   * `stream` just before stage i is enqueued (the last one after the last
+   * stage). Stages: proxies, softmax pass, normaliser merge, mass pass, mass
+   * sum, coverage vote, top-k, gather; a stage that does not run records its
+   * event next to its neighbour's. */
+  void** stage_events;
+  int32_t n_stage_events;
+  int32_t launches;   /* out: number of kernels the call enqueued */
+  int32_t score_path; /* out: 1 if steps 2-4 ran on the tensor cores (tcgen05),
+                         0 if on the CUDA cores (fp32 FMA) */
 } mmshift_debug;
+
+#define MMSHIFT_N_STAGES 8
 
 /* Fill *p with the paper's default hyper-parameters (Section 4.1). */
 void mmshift_default_params(mmshift_params* p);

@@ -55,10 +55,16 @@ class Shape(ctypes.Structure):
     ]
 
 
+MMSHIFT_N_STAGES = 8
+STAGES = ("proxies", "softmax_pass", "merge", "mass_pass", "mass_sum", "cover", "topk", "gather")
+
+
 class Debug(ctypes.Structure):
     _fields_ = [
         ("proxies", ctypes.c_void_p), ("group_mass", ctypes.c_void_p), ("anchor", ctypes.c_void_p),
         ("mass", ctypes.c_void_p), ("scores", ctypes.c_void_p),
+        ("stage_events", ctypes.POINTER(ctypes.c_void_p)), ("n_stage_events", ctypes.c_int32),
+        ("launches", ctypes.c_int32), ("score_path", ctypes.c_int32),
     ]
 
 
@@ -210,6 +216,14 @@ def mmshift_poll_status(workspace, stream=None) -> int:
     return load_library().mmshift_poll_status(_ptr(workspace), _ptr(stream))
 
 
-def make_debug(proxies=None, group_mass=None, anchor=None, mass=None, scores=None) -> Debug:
-    return Debug(proxies=_ptr(proxies), group_mass=_ptr(group_mass), anchor=_ptr(anchor),
-                 mass=_ptr(mass), scores=_ptr(scores))
+def make_debug(proxies=None, group_mass=None, anchor=None, mass=None, scores=None,
+               stage_events=None) -> Debug:
+    """stage_events: sequence of MMSHIFT_N_STAGES + 1 torch.cuda.Event (timing)."""
+    dbg = Debug(proxies=_ptr(proxies), group_mass=_ptr(group_mass), anchor=_ptr(anchor),
+                mass=_ptr(mass), scores=_ptr(scores))
+    if stage_events is not None:
+        arr = (ctypes.c_void_p * len(stage_events))(*[e.cuda_event for e in stage_events])
+        dbg.stage_events = arr
+        dbg.n_stage_events = len(stage_events)
+        dbg._keep = arr
+    return dbg

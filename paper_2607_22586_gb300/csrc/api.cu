@@ -174,13 +174,44 @@ mmshift_status prepare(const mmshift_shape* s, const mmshift_params* p, Problem*
   return build_problem(s, p, P);
 }
 
+// Records stage-boundary events when the caller asked for them.
+struct StageMarks {
+  cudaEvent_t* ev = nullptr;
+  cudaStream_t st = nullptr;
+  cudaError_t mark(int stage) const {
+    return ev ? cudaEventRecord(ev[stage], st) : cudaSuccess;
+  }
+};
+
+StageMarks marks_of(const mmshift_debug* dbg, cudaStream_t st) {
+  StageMarks m;
+  m.st = st;
+  if (dbg && dbg->stage_events && dbg->n_stage_events >= MMSHIFT_N_STAGES + 1)
+    m.ev = reinterpret_cast<cudaEvent_t*>(dbg->stage_events);
+  return m;
+}
+
+// Kernels one mmshift_select call enqueues (reported through mmshift_debug).
+int count_launches(const Problem& P, const Buffers& bf) {
+  int n = 1;                                   // proxies
+  n += umma_supported(P) ? umma_launches(P) : 3;  // softmax pass, merge, mass pass
+  if (bf.mass && P.total_T) n += 1;            // mass sum
+  if (P.mode == MMSHIFT_SCORE_VOTE && P.G) n += 1;  // coverage vote
+  n += 1;                                      // top-k
+  if (P.R) n += 1;                             // gather
+  return n;
+}
+
 // Proxies (sampled or given) packed into the workspace, then steps 2-4.
 mmshift_status run_mass(const Problem& P, const Buffers& bf, const void* K, const void* qwin,
-                        cudaStream_t st) {
-  cudaError_t e = launch_proxy_pack(P, bf, st, qwin);
+                        cudaStream_t st, const StageMarks& mk = StageMarks()) {
+  cudaError_t e;
+  if ((e = mk.mark(0)) != cudaSuccess) return cuda_fail(e);
+  if ((e = launch_proxy_pack(P, bf, st, qwin)) != cudaSuccess) return cuda_fail(e);
+  e = umma_supported(P) ? launch_score_umma(P, bf, st, K, mk.ev)
+                        : launch_score_simt(P, bf, st, K, mk.ev);
   if (e != cudaSuccess) return cuda_fail(e);
-  e = umma_supported(P) ? launch_score_umma(P, bf, st, K) : launch_score_simt(P, bf, st, K);
-  if (e != cudaSuccess) return cuda_fail(e);
+  if ((e = mk.mark(4)) != cudaSuccess) return cuda_fail(e);
   if ((e = launch_mass_sum(P, bf, st)) != cudaSuccess) return cuda_fail(e);
   return MMSHIFT_OK;
 }
@@ -328,11 +359,19 @@ mmshift_status mmshift_select(const mmshift_shape* s, const void* K, const void*
     bf.mass = dbg->mass;
   }
   const cudaStream_t cs = (cudaStream_t)stream;
-  if ((st = run_mass(P, bf, K, Qwin, cs)) != MMSHIFT_OK) return st;
-  cudaError_t e = cudaSuccess;
-  if (P.mode == MMSHIFT_SCORE_VOTE) e = launch_cover(P, bf, cs);
+  const StageMarks mk = marks_of(dbg, cs);
+  if ((st = run_mass(P, bf, K, Qwin, cs, mk)) != MMSHIFT_OK) return st;
+  cudaError_t e = mk.mark(5);
+  if (e == cudaSuccess && P.mode == MMSHIFT_SCORE_VOTE) e = launch_cover(P, bf, cs);
+  if (e == cudaSuccess) e = mk.mark(6);
   if (e == cudaSuccess) e = launch_topk(P, bf, cs, out_idx, false);
+  if (e == cudaSuccess) e = mk.mark(7);
   if (e == cudaSuccess) e = launch_gather(P, bf, cs, K, V, out_idx, out_K, out_V);
+  if (e == cudaSuccess) e = mk.mark(8);
+  if (dbg) {
+    const_cast<mmshift_debug*>(dbg)->launches = count_launches(P, bf);
+    const_cast<mmshift_debug*>(dbg)->score_path = umma_supported(P) ? 1 : 0;
+  }
   return e == cudaSuccess ? MMSHIFT_OK : cuda_fail(e);
 }
 

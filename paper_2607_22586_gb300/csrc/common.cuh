@@ -115,11 +115,14 @@ __device__ __forceinline__ void set_status(int* status, int bit) {
 // Host-side launchers (one translation unit each).
 cudaError_t launch_proxy_pack(const Problem& P, const Buffers& bf, cudaStream_t st,
                               const void* qwin);
+// ev (nullable): stage events 1 (softmax pass), 2 (merge) and 3 (mass pass)
+// are recorded just before the corresponding launch.
 cudaError_t launch_score_simt(const Problem& P, const Buffers& bf, cudaStream_t st,
-                              const void* K);
+                              const void* K, cudaEvent_t* ev);
 cudaError_t launch_score_umma(const Problem& P, const Buffers& bf, cudaStream_t st,
-                              const void* K);
+                              const void* K, cudaEvent_t* ev);
 bool umma_supported(const Problem& P);
+int umma_launches(const Problem& P);
 cudaError_t launch_merge(const Problem& P, const Buffers& bf, cudaStream_t st);
 cudaError_t launch_cover(const Problem& P, const Buffers& bf, cudaStream_t st);
 cudaError_t launch_mass_sum(const Problem& P, const Buffers& bf, cudaStream_t st);

@@ -32,9 +32,31 @@ __device__ __forceinline__ void philox4x64_10(uint64_t c[4], uint64_t k0, uint64
   }
 }
 
-// uint64 -> uniform in (0, 1]: ((x >> 11) + 1/2) * 2^-53, rounded to float.
-__device__ __forceinline__ float uniform_of(uint64_t x) {
-  return (__ull2float_rn(x >> 11) + 0.5f) * 1.1102230246251565e-16f;
+// Box-Muller on two Philox words a, c: with u = ((a >> 11) + 1/2) 2^-53 and
+// v = ((c >> 11) + 1/2) 2^-53, returns sqrt(-2 ln u) (cos 2 pi v, sin 2 pi v).
+// Evaluated in float32 without losing the precision the 53-bit uniforms carry
+// where it matters: ln u for u >= 1/2 is log1p(-(1 - u)) with 1 - u taken from
+// the integer complement, and the angle is first reduced to (-1/2, 1/2] turn in
+// integer arithmetic, so sin/cos near their zeros keep full relative precision.
+__device__ __forceinline__ void box_muller(uint64_t a, uint64_t c, float& z0, float& z1) {
+  constexpr float k2m53 = 1.1102230246251565e-16f;  // 2^-53
+  constexpr float k2m52 = 2.220446049250313e-16f;   // 2^-52
+  const uint64_t ma = a >> 11;
+  float lnu;
+  if (ma < (1ull << 52)) {
+    lnu = logf((__ull2float_rn(ma) + 0.5f) * k2m53);
+  } else {
+    const uint64_t comp = ((1ull << 53) - 1) - ma;
+    lnu = log1pf(-(__ull2float_rn(comp) + 0.5f) * k2m53);
+  }
+  const float r = sqrtf(-2.0f * lnu);
+  const uint64_t mc = c >> 11;
+  const int64_t cen = (int64_t)mc - (mc >= (1ull << 52) ? (int64_t)(1ull << 53) : 0);
+  const float two_v = (__ll2float_rn(cen) + 0.5f) * k2m52;  // 2v reduced to (-1, 1]
+  float sv, cv;
+  sincospif(two_v, &sv, &cv);
+  z0 = r * cv;
+  z1 = r * sv;
 }
 
 // Four standard normals for dims 4q..4q+3 of proxy i of query head hq.
@@ -43,13 +65,8 @@ __device__ __forceinline__ void normals4(const Problem& P, int i, int q, int hq,
   uint64_t c[4] = {(uint64_t)i * (uint64_t)(P.d / 4) + (uint64_t)q, (uint64_t)hq,
                    (uint64_t)b, (uint64_t)(int64_t)layer};
   philox4x64_10(c, P.seed, 0ull);
-  const float u0 = uniform_of(c[0]), u1 = uniform_of(c[1]);
-  const float u2 = uniform_of(c[2]), u3 = uniform_of(c[3]);
-  const float r01 = sqrtf(-2.0f * logf(u0)), r23 = sqrtf(-2.0f * logf(u2));
-  float s1, c1, s3, c3;
-  sincospif(2.0f * u1, &s1, &c1);
-  sincospif(2.0f * u3, &s3, &c3);
-  z[0] = r01 * c1; z[1] = r01 * s1; z[2] = r23 * c3; z[3] = r23 * s3;
+  box_muller(c[0], c[1], z[0], z[1]);
+  box_muller(c[2], c[3], z[2], z[3]);
 }
 
 template <typename T, int D>

@@ -201,7 +201,8 @@ __global__ void __launch_bounds__(256) pass2_simt(Problem P, Buffers bf, const T
 }
 
 template <typename T, int D>
-cudaError_t launch_t(const Problem& P, const Buffers& bf, cudaStream_t st, const void* K) {
+cudaError_t launch_t(const Problem& P, const Buffers& bf, cudaStream_t st, const void* K,
+                     cudaEvent_t* ev) {
   const size_t sm1 = (2 * TILE * (D + 1) + TILE * (TILE + 1)) * sizeof(float);
   const size_t sm2 = sm1 + (TILE + (size_t)(P.G + 1) * TILE) * sizeof(float);
   cudaError_t e;
@@ -210,9 +211,12 @@ cudaError_t launch_t(const Problem& P, const Buffers& bf, cudaStream_t st, const
   if ((e = cudaFuncSetAttribute(pass2_simt<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)sm2)) != cudaSuccess) return e;
   dim3 g1(P.Hkv * P.total_splits * (P.Prows_pad / TILE), P.L);
+  if (ev && (e = cudaEventRecord(ev[1], st)) != cudaSuccess) return e;
   pass1_simt<T, D><<<g1, 256, sm1, st>>>(P, bf, (const T*)K);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if (ev && (e = cudaEventRecord(ev[2], st)) != cudaSuccess) return e;
   if ((e = launch_merge(P, bf, st)) != cudaSuccess) return e;
+  if (ev && (e = cudaEventRecord(ev[3], st)) != cudaSuccess) return e;
   int tiles = 0;
   for (int b = 0; b < P.B; ++b) tiles += (P.req[b].t_len + TILE - 1) / TILE;
   dim3 g2(P.Hkv * tiles, P.L);
@@ -229,11 +233,12 @@ cudaError_t launch_merge(const Problem& P, const Buffers& bf, cudaStream_t st) {
 }
 
 cudaError_t launch_score_simt(const Problem& P, const Buffers& bf, cudaStream_t st,
-                              const void* K) {
+                              const void* K, cudaEvent_t* ev) {
   if (P.dtype == MMSHIFT_BF16)
-    return P.d == 128 ? launch_t<__nv_bfloat16, 128>(P, bf, st, K)
-                      : launch_t<__nv_bfloat16, 64>(P, bf, st, K);
-  return P.d == 128 ? launch_t<float, 128>(P, bf, st, K) : launch_t<float, 64>(P, bf, st, K);
+    return P.d == 128 ? launch_t<__nv_bfloat16, 128>(P, bf, st, K, ev)
+                      : launch_t<__nv_bfloat16, 64>(P, bf, st, K, ev);
+  return P.d == 128 ? launch_t<float, 128>(P, bf, st, K, ev)
+                    : launch_t<float, 64>(P, bf, st, K, ev);
 }
 
 }  // namespace mmshift

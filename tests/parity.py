@@ -155,7 +155,7 @@ def uncertain_votes(abar: np.ndarray, tau: float) -> np.ndarray:
     return unc
 
 
-def check_request(gpu, ref, h, lo, hi, layer, what=""):
+def check_request(gpu, ref, h, lo, hi, layer, what="", out_lo=0):
     """Compare one request of one layer: masses, anchor, votes, scores, selection, gather."""
     G, tau, lam, mode = h["n_groups"], h["tau"], h["lam"], h["score_mode"]
     hkv = ref["anchor"].shape[0]
@@ -176,7 +176,7 @@ def check_request(gpu, ref, h, lo, hi, layer, what=""):
             assert np.all(dv <= unc.sum(axis=0)), f"{what} head {hh}: vote mismatch outside band"
     dev_max = np.max(np.abs(s_gpu - s_ref)) if T else 0.0
     keep_rows = ref["idx"].shape[0]
-    idx_gpu = gpu["idx"][layer]
+    idx_gpu = gpu["idx"][layer][out_lo:out_lo + keep_rows]
     for hh in range(hkv):
         got = idx_gpu[:, hh]
         assert got.shape[0] == keep_rows

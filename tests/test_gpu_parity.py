@@ -30,7 +30,7 @@ def _check_all(wl, gpu, refs, h, layer=0, what=""):
     for b, lo, hi, olo in _requests(wl):
         if refs[b] is None:
             continue
-        PT.check_request(gpu, refs[b], h, lo, hi, layer, f"{what} req {b}")
+        PT.check_request(gpu, refs[b], h, lo, hi, layer, f"{what} req {b}", out_lo=olo)
         PT.check_gather(gpu, wl, layer, lo, olo, min(wl.budgets[b], hi - lo), hi - lo, wl.n_kv_heads)
 
 
@@ -53,15 +53,20 @@ def test_proxies_match_oracle(name, rope):
         z = O.proxy_normals(h["seed"], h["layer_id"], b, wl.n_q_heads, h["n_proxies"], wl.head_dim)
         ref = O.build_proxies(li.Qwin[b], z, h["gamma"], wl.seq_lens[b], wl.dtype, rope,
                               h["rope_pos_offset"])
+        # fp32 sampling vs fp64: the pre-rounding error is bounded relative to
+        # the magnitude of the two terms mu and gamma*sigma*z, not to their
+        # (possibly cancelling) sum; rounding to bf16 adds at most one ulp
+        mu, sig = O.window_stats(li.Qwin[b])
+        scale = np.abs(mu)[:, None, :] + h["gamma"] * sig[:, None, :] * (1.0 + np.abs(z))
+        diff = np.abs(got[b] - ref)
         if wl.dtype == S.BF16:
             _, e = np.frexp(np.maximum(np.abs(ref), np.abs(got[b])))
             ulp = np.ldexp(1.0, e - 8)
-            diff = np.abs(got[b] - ref)
-            assert np.all(diff <= ulp * 1.0001), "bf16 proxies off by more than one ulp"
+            assert np.all(diff <= ulp + 2e-6 * scale), "bf16 proxies off by more than one ulp"
             frac = np.mean(diff > 0)
-            assert frac <= 1e-3, f"{frac:.2e} of proxies differ by one ulp"
+            assert frac <= 1e-3, f"{frac:.2e} of proxies differ"
         else:
-            np.testing.assert_allclose(got[b], ref, rtol=4e-6, atol=1e-6)
+            assert np.all(diff <= 2e-6 * scale), f"max scaled error {np.max(diff / scale):.3g}"
 
 
 # ---------------------------------------------------------------------------
