@@ -200,6 +200,37 @@ mmshift_status mmshift_select(const mmshift_shape* s, const void* K, const void*
                               void* out_V, const mmshift_debug* dbg, void* workspace,
                               size_t workspace_bytes, mmshift_stream_t stream);
 
+/* Allocation-free variant of mmshift_scores_topk.
+ *
+ * The paper has no counterpart: this entry point exists for callers that
+ * cannot allocate device memory -- e.g. code running inside a runtime or
+ * plugin host that owns every device allocation and hands out no workspace,
+ * or a serving loop whose memory plan is frozen after start-up. Instead of a
+ * caller workspace it uses a scratch array compiled into the library: a
+ * file-scope __device__ array of MMSHIFT_NOALLOC_SCRATCH_BYTES (8 MiB) that
+ * every GPU which loads the library holds until the process exits. It calls
+ * no cudaMalloc/cudaFree and no allocating library routine.
+ *
+ *  - Inputs and outputs are the caller's, exactly as in mmshift_scores_topk
+ *    (group_mass, anchor, nullable scores, out_idx).
+ *  - Scratch use is L*Hkv*G*ceil32(T_b)/8 bytes of coverage bitmaps, plus
+ *    L*Hkv*T*4 bytes of scores when `scores` is NULL (each part rounded up to
+ *    256 bytes). Larger problems are rejected with MMSHIFT_ERR_WORKSPACE before
+ *    anything is enqueued.
+ *  - The first call on a device (with that device current) looks up the
+ *    array's device address with cudaGetSymbolAddress; make that first call
+ *    before any stream capture on that device.
+ *  - Every call on a device shares the one array, which keeps the contents of
+ *    the last call; nothing in it needs to start at zero (every byte read is
+ *    first written by the same call). Calls whose work overlaps on the GPU --
+ *    on different streams, or from different host threads without ordering --
+ *    race on the array and must be serialised by the caller. */
+#define MMSHIFT_NOALLOC_SCRATCH_BYTES (8u << 20)
+mmshift_status mmshift_scores_topk_noalloc(const mmshift_shape* s, const mmshift_params* p,
+                                           const float* group_mass, const float* anchor,
+                                           float* scores, int32_t* out_idx,
+                                           mmshift_stream_t stream);
+
 /* Synchronise `stream`, read and clear the device status word kept in the
  * workspace: MMSHIFT_OK, MMSHIFT_ERR_TIMEOUT or MMSHIFT_ERR_DEVICE. */
 mmshift_status mmshift_poll_status(void* workspace, mmshift_stream_t stream);

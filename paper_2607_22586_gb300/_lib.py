@@ -31,8 +31,9 @@ EXPORTED = [
     "mmshift_default_params", "mmshift_output_rows", "mmshift_workspace_size",
     "mmshift_build_proxies", "mmshift_proxy_mass", "mmshift_scores_topk", "mmshift_topk",
     "mmshift_gather", "mmshift_select", "mmshift_poll_status", "mmshift_status_string",
-    "mmshift_last_cuda_error",
+    "mmshift_last_cuda_error", "mmshift_scores_topk_noalloc",
 ]
+MMSHIFT_NOALLOC_SCRATCH_BYTES = 8 << 20
 
 
 class Params(ctypes.Structure):
@@ -104,6 +105,8 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.mmshift_select.argtypes = [_SP, _VP, _VP, _VP, _VP, _PP, _VP, _VP, _VP,
                                    ctypes.POINTER(Debug), _VP, ctypes.c_size_t, _VP]
     lib.mmshift_select.restype = st
+    lib.mmshift_scores_topk_noalloc.argtypes = [_SP, _PP, _VP, _VP, _VP, _VP, _VP]
+    lib.mmshift_scores_topk_noalloc.restype = st
     lib.mmshift_poll_status.argtypes = [_VP, _VP]
     lib.mmshift_poll_status.restype = st
     lib.mmshift_status_string.argtypes = [st]
@@ -191,6 +194,15 @@ def mmshift_scores_topk(shape, params, group_mass, anchor, scores, out_idx, work
     return load_library().mmshift_scores_topk(
         ctypes.byref(shape), ctypes.byref(params), _ptr(group_mass), _ptr(anchor), _ptr(scores),
         _ptr(out_idx), _ptr(workspace), workspace_bytes, _ptr(stream))
+
+
+def mmshift_scores_topk_noalloc(shape, params, group_mass, anchor, scores, out_idx,
+                                stream=None) -> int:
+    """Allocation-free vote + top-k: scratch comes from a static device array
+    inside the library (for callers that cannot allocate device memory)."""
+    return load_library().mmshift_scores_topk_noalloc(
+        ctypes.byref(shape), ctypes.byref(params), _ptr(group_mass), _ptr(anchor), _ptr(scores),
+        _ptr(out_idx), _ptr(stream))
 
 
 def mmshift_topk(shape, scores, out_idx, workspace, workspace_bytes, stream=None) -> int:

@@ -218,6 +218,14 @@ mmshift_status run_mass(const Problem& P, const Buffers& bf, const void* K, cons
 
 }  // namespace
 
+namespace mmshift {
+// Shared with the allocation-free entry point (noalloc.cu).
+mmshift_status noalloc_prepare(const mmshift_shape* s, const mmshift_params* p, Problem* P) {
+  return prepare(s, p, P);
+}
+mmshift_status noalloc_cuda_fail(cudaError_t e) { return cuda_fail(e); }
+}  // namespace mmshift
+
 extern "C" {
 
 void mmshift_default_params(mmshift_params* p) {
