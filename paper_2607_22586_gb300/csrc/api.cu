@@ -191,10 +191,16 @@ StageMarks marks_of(const mmshift_debug* dbg, cudaStream_t st) {
   return m;
 }
 
+// Tensor-core scoring when the device, dtype, shape and K's alignment (TMA
+// needs a 16-byte aligned base) allow it; CUDA-core scoring otherwise.
+int choose_umma(const Problem& P, const void* K) {
+  return (umma_supported(P) && (reinterpret_cast<uintptr_t>(K) & 15) == 0) ? 1 : 0;
+}
+
 // Kernels one mmshift_select call enqueues (reported through mmshift_debug).
 int count_launches(const Problem& P, const Buffers& bf) {
   int n = 1;                                   // proxies
-  n += umma_supported(P) ? umma_launches(P) : 3;  // softmax pass, merge, mass pass
+  n += P.use_umma ? umma_launches(P) : 3;      // softmax pass, merge, mass pass
   if (bf.mass && P.total_T) n += 1;            // mass sum
   if (P.mode == MMSHIFT_SCORE_VOTE && P.G) n += 1;  // coverage vote
   n += 1;                                      // top-k
@@ -208,8 +214,8 @@ mmshift_status run_mass(const Problem& P, const Buffers& bf, const void* K, cons
   cudaError_t e;
   if ((e = mk.mark(0)) != cudaSuccess) return cuda_fail(e);
   if ((e = launch_proxy_pack(P, bf, st, qwin)) != cudaSuccess) return cuda_fail(e);
-  e = umma_supported(P) ? launch_score_umma(P, bf, st, K, mk.ev)
-                        : launch_score_simt(P, bf, st, K, mk.ev);
+  e = P.use_umma ? launch_score_umma(P, bf, st, K, mk.ev)
+                 : launch_score_simt(P, bf, st, K, mk.ev);
   if (e != cudaSuccess) return cuda_fail(e);
   if ((e = mk.mark(4)) != cudaSuccess) return cuda_fail(e);
   if ((e = launch_mass_sum(P, bf, st)) != cudaSuccess) return cuda_fail(e);
@@ -289,6 +295,7 @@ mmshift_status mmshift_proxy_mass(const mmshift_shape* s, const void* K, const v
   mmshift_status st = prepare(s, p, &P);
   if (st != MMSHIFT_OK) return st;
   if (!p || !K || !Qwin || !anchor || (P.G && !group_mass)) return MMSHIFT_ERR_INVALID_ARG;
+  P.use_umma = choose_umma(P, K);
   Buffers bf;
   if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
   bf.proxies_in = proxies;
@@ -356,6 +363,7 @@ mmshift_status mmshift_select(const mmshift_shape* s, const void* K, const void*
   mmshift_status st = prepare(s, p, &P);
   if (st != MMSHIFT_OK) return st;
   if (!p || !K || !V || !Qwin || !out_idx || !out_K || !out_V) return MMSHIFT_ERR_INVALID_ARG;
+  P.use_umma = choose_umma(P, K);
   Buffers bf;
   if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
   bf.proxies_in = proxies_in;
@@ -378,7 +386,7 @@ mmshift_status mmshift_select(const mmshift_shape* s, const void* K, const void*
   if (e == cudaSuccess) e = mk.mark(8);
   if (dbg) {
     const_cast<mmshift_debug*>(dbg)->launches = count_launches(P, bf);
-    const_cast<mmshift_debug*>(dbg)->score_path = umma_supported(P) ? 1 : 0;
+    const_cast<mmshift_debug*>(dbg)->score_path = P.use_umma ? 1 : 0;
   }
   return e == cudaSuccess ? MMSHIFT_OK : cuda_fail(e);
 }

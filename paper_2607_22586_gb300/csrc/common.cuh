@@ -11,7 +11,7 @@ namespace mmshift {
 
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr int kChunk = 16;       // proxy rows per packing chunk (one group id)
-constexpr int kRowTile = 128;    // proxy rows are padded to a multiple of this
+constexpr int kRowTile = 256;    // proxy rows are padded to a multiple of this
 
 // Status bits the kernels OR into the workspace status word.
 enum : int {
@@ -47,6 +47,7 @@ struct Problem {
   int32_t layer_id0;
   float rope_theta;
   int32_t rope_off;
+  int32_t use_umma;    // steps 2-4 on the tensor cores (set per call)
   ReqInfo req[MMSHIFT_MAX_BATCH];
 };
 

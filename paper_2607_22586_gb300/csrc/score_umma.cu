@@ -1,15 +1,511 @@
-// Steps 2-4 on the 5th-generation tensor cores (tcgen05 + TMA + TMEM).
+// Steps 2-4 on the 5th-generation tensor cores (tcgen05 + TMA + TMEM), bf16:
+// proxy logits, row softmax over the whole prompt and group-mass aggregation
+// (Section 3.2.2; Appendix B).
+//
+// Both passes are one persistent, warp-specialised kernel (one CTA per SM):
+//   warp 0      TMA producer: a stationary block of up to 256 packed proxy rows
+//               (reloaded only when the (layer, request, KV head, block) of
+//               the work unit changes) and a 4-stage ring of 128-key K tiles;
+//   warp 1      TMEM allocator and MMA issuer (one thread): d/16 tcgen05.mma
+//               of K = 16 per key tile into one of two TMEM accumulators;
+//   warps 2-9   epilogue (two warpgroups): tcgen05.ld of the accumulator,
+//               exp2 and reductions in registers, outputs to global memory.
+// Work units are (layer, request, KV head, proxy block, key split of 1024
+// keys), split fastest; each CTA takes a contiguous range of units, so the
+// stationary block changes rarely and the split boundaries (and so the
+// merge order of the softmax partials) are those of the CUDA-core path.
+//
+// Softmax pass (PASS 1): stationary = 2 x 128 proxy rows as the M operand,
+//   K tile = N operand (M=128, N=128, two MMAs); the accumulator lane is a
+//   proxy row, so each thread keeps its row's running (max, sum of exp2) over
+//   the 128 keys of a tile without any cross-thread reduction. The running max
+//   is only raised when a 32-key chunk's sum would exceed 2^64 (or on the
+//   first chunk), so the common path is one FFMA, one MUFU.EX2 and one FADD
+//   per logit.
+// Mass pass (PASS 2): K tile = M operand (128 keys), stationary = up to 256
+//   proxy rows holding whole groups as the N operand; the accumulator lane is
+//   a key, so each thread sums exp2(x - c_row) over the columns of a group in
+//   registers and writes one group mass per key (coalesced along keys).
+// Every wait is bounded; a CTA that gives up raises the timeout status bit,
+// stops issuing work and still frees its TMEM.
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
 #include "common.cuh"
+#include "umma.cuh"
 
 namespace mmshift {
+namespace {
 
-bool umma_supported(const Problem& P) { (void)P; return false; }
+using namespace umma;
+
+constexpr int BK = 128;          // keys per K tile
+constexpr int SROWS = 256;       // stationary proxy rows per block
+constexpr int NSTAGE = 4;        // K-tile ring depth
+constexpr int NTHREADS = 320;
+constexpr int EPI_WARP0 = 2;
+constexpr int NEPI = 256;        // epilogue threads
+constexpr int TMEM_COLS = 512;
+constexpr int ACC_STRIDE = 256;  // TMEM columns per accumulator buffer
+
+struct Sched {
+  int32_t uoff[MMSHIFT_MAX_BATCH + 1];  // per-layer units, prefix over requests
+  int32_t ntiles;                        // stationary blocks per (request, KV head)
+  int32_t units;                         // total units of the launch
+  int32_t gpt;                           // mass pass: groups per regular block
+  int32_t n_reg;                         // mass pass: regular blocks
+  int32_t anchor_merged;                 // mass pass: anchor rows ride on the last block
+};
+
+struct Unit {
+  int l, b, h, tile, split, t0, t1;
+};
+
+__device__ __forceinline__ Unit decode(const Problem& P, const Sched& S, int u) {
+  Unit x;
+  const int per_layer = S.uoff[P.B];
+  x.l = u / per_layer;
+  int r = u - x.l * per_layer;
+  int b = 0;
+  while (b + 1 < P.B && S.uoff[b + 1] <= r) ++b;
+  x.b = b;
+  r -= S.uoff[b];
+  const int ns = P.req[b].nsplit;
+  x.split = r % ns;
+  r /= ns;
+  x.tile = r % S.ntiles;
+  x.h = r / S.ntiles;
+  x.t0 = x.split * P.split_len;
+  x.t1 = min(P.req[b].t_len, x.t0 + P.split_len);
+  return x;
+}
+
+// Rows of stationary block t of the mass pass.
+struct Block {
+  int row0, rows, g0, ng, anchor;
+};
+
+__host__ __device__ inline Block mass_block(const Problem& P, const Sched& S, int t) {
+  Block k;
+  if (t < S.n_reg) {
+    k.g0 = t * S.gpt;
+    k.ng = min(P.G - k.g0, S.gpt);
+    k.row0 = k.g0 * P.RG;
+    k.rows = k.ng * P.RG;
+    k.anchor = (S.anchor_merged && t == S.n_reg - 1) ? 1 : 0;
+    if (k.anchor) k.rows += P.anchor_rows;
+  } else {
+    k.g0 = P.G;
+    k.ng = 0;
+    k.row0 = P.n_group_rows;
+    k.rows = P.anchor_rows;
+    k.anchor = 1;
+  }
+  return k;
+}
+
+__device__ __forceinline__ long long block_key(const Problem& P, const Sched& S, const Unit& x) {
+  return ((long long)(x.l * P.B + x.b) * P.Hkv + x.h) * S.ntiles + x.tile;
+}
+
+template <int D>
+struct Smem {
+  static constexpr int CH = D / 64;                         // 128-byte K chunks
+  static constexpr int STAT_BYTES = CH * SROWS * 128;
+  static constexpr int STAGE_BYTES = CH * BK * 128;
+  static constexpr int RING_BYTES = NSTAGE * STAGE_BYTES;
+  static constexpr int DYN_BYTES = 1024 + STAT_BYTES + RING_BYTES;
+};
+
+// Sum over the RG (multiple of 16) accumulator columns of one group:
+// sum_j exp2(acc_j * alpha - c_j), four partial sums added in a fixed order.
+__device__ __forceinline__ float group_sum(uint32_t tcol, const float* __restrict__ c, int ncols,
+                                           float alpha) {
+  float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+  for (int cc = 0; cc < ncols; cc += 16) {
+    float v[16];
+    tmem_ld16(tcol + cc, v);
+    const float4* c4 = reinterpret_cast<const float4*>(c + cc);
+    float cv[16];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float4 t = __ldg(c4 + i);
+      cv[4 * i] = t.x; cv[4 * i + 1] = t.y; cv[4 * i + 2] = t.z; cv[4 * i + 3] = t.w;
+    }
+    tmem_wait_ld();
+#pragma unroll
+    for (int j = 0; j < 16; j += 4) {
+      a0 += fast_exp2(fmaf(v[j], alpha, -cv[j]));
+      a1 += fast_exp2(fmaf(v[j + 1], alpha, -cv[j + 1]));
+      a2 += fast_exp2(fmaf(v[j + 2], alpha, -cv[j + 2]));
+      a3 += fast_exp2(fmaf(v[j + 3], alpha, -cv[j + 3]));
+    }
+  }
+  return (a0 + a1) + (a2 + a3);
+}
+
+template <int PASS, int D>
+__global__ void __launch_bounds__(NTHREADS, 1)
+    score_umma_kernel(const __grid_constant__ CUtensorMap kmap,
+                      const __grid_constant__ CUtensorMap pmap, const __grid_constant__ Problem P,
+                      const __grid_constant__ Sched S, Buffers bf) {
+  using SM = Smem<D>;
+  extern __shared__ unsigned char smraw[];
+  unsigned char* sm =
+      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
+  unsigned char* stat = sm;
+  unsigned char* ring = sm + SM::STAT_BYTES;
+  __shared__ uint64_t full[NSTAGE], empty[NSTAGE], sfull, sempty, tfull[2], tempty[2];
+  __shared__ uint32_t tbase;
+  __shared__ int abort_flag;
+  volatile int* abort_ = &abort_flag;
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int u_begin = (int)((long long)blockIdx.x * S.units / gridDim.x);
+  const int u_end = (int)((long long)(blockIdx.x + 1) * S.units / gridDim.x);
+
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    for (int s = 0; s < NSTAGE; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(&sfull, 1);
+    mbar_init(&sempty, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&tfull[i], 1);
+      mbar_init(&tempty[i], NEPI);
+    }
+    fence_barrier_init();
+    prefetch_tmap(&kmap);
+    prefetch_tmap(&pmap);
+  }
+  if (warp == 1) {
+    tmem_alloc(&tbase, TMEM_COLS);
+    tmem_relinquish();
+  }
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem = tbase;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0, sphase = 0;
+      long long prev = -1;
+      for (int u = u_begin; u < u_end; ++u) {
+        const Unit x = decode(P, S, u);
+        const long long key = block_key(P, S, x);
+        if (key != prev) {
+          if (!mbar_wait(&sempty, sphase ^ 1u, abort_)) break;
+          int row0, rows;
+          if (PASS == 1) {
+            row0 = x.tile * SROWS;
+            rows = SROWS;
+          } else {
+            const Block k = mass_block(P, S, x.tile);
+            row0 = k.row0;
+            rows = k.rows;
+          }
+          mbar_expect_tx(&sfull, (uint32_t)(rows * D * 2));
+          const int zc = (x.l * P.B + x.b) * P.Hkv + x.h;
+          for (int c = 0; c < SM::CH; ++c)
+            for (int r = 0; r < rows; r += 16)
+              tma_load_3d(stat + c * SROWS * 128 + r * 128, &pmap, &sfull, c * 64, row0 + r, zc);
+          sphase ^= 1u;
+          prev = key;
+        }
+        const int kbase = P.req[x.b].tok_off;
+        bool ok = true;
+        for (int kt = x.t0; kt < x.t1; kt += BK) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_)) { ok = false; break; }
+          mbar_expect_tx(&full[stage], (uint32_t)SM::STAGE_BYTES);
+          for (int c = 0; c < SM::CH; ++c)
+            tma_load_3d(ring + stage * SM::STAGE_BYTES + c * BK * 128, &kmap, &full[stage],
+                        x.h * D + c * 64, kbase + kt, x.l);
+          if (++stage == NSTAGE) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      int stage = 0, buf = 0;
+      uint32_t phase = 0, bphase = 0, sphase = 0;
+      long long prev = -1;
+      uint32_t idesc = idesc_bf16_f32(128, 128);
+      for (int u = u_begin; u < u_end; ++u) {
+        const Unit x = decode(P, S, u);
+        const long long key = block_key(P, S, x);
+        if (key != prev) {
+          if (prev != -1) mma_commit(&sempty);   // old block free once its MMAs finish
+          if (!mbar_wait(&sfull, sphase, abort_)) break;
+          sphase ^= 1u;
+          fence_after();
+          if (PASS == 2) idesc = idesc_bf16_f32(128, mass_block(P, S, x.tile).rows);
+          prev = key;
+        }
+        bool ok = true;
+        for (int kt = x.t0; kt < x.t1; kt += BK) {
+          if (!mbar_wait(&full[stage], phase, abort_) ||
+              !mbar_wait(&tempty[buf], bphase ^ 1u, abort_)) { ok = false; break; }
+          fence_after();
+          const uint32_t ks_base = smem_u32(ring + stage * SM::STAGE_BYTES);
+          const uint32_t st_base = smem_u32(stat);
+          const uint32_t dcol = tmem + (uint32_t)(buf * ACC_STRIDE);
+#pragma unroll
+          for (int ks = 0; ks < D / 16; ++ks) {
+            const int c = ks / 4, w = ks % 4;
+            const uint64_t kd = sdesc_k_sw128(ks_base + c * BK * 128 + w * 32);
+            if (PASS == 1) {
+#pragma unroll
+              for (int m = 0; m < 2; ++m) {
+                const uint64_t pd = sdesc_k_sw128(st_base + c * SROWS * 128 + m * 128 * 128 + w * 32);
+                mma_bf16(dcol + m * 128, pd, kd, idesc, ks > 0 ? 1u : 0u);
+              }
+            } else {
+              const uint64_t pd = sdesc_k_sw128(st_base + c * SROWS * 128 + w * 32);
+              mma_bf16(dcol, kd, pd, idesc, ks > 0 ? 1u : 0u);
+            }
+          }
+          mma_commit(&empty[stage]);
+          mma_commit(&tfull[buf]);
+          if (++stage == NSTAGE) { stage = 0; phase ^= 1u; }
+          buf ^= 1;
+          if (buf == 0) bphase ^= 1u;
+        }
+        if (!ok) break;
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int ew = warp - EPI_WARP0;      // 0..7
+    const int wg = ew / 4;                // warpgroup
+    const int q = warp % 4;               // TMEM lane quarter this warp may access
+    const int lrow = q * 32 + lane;       // accumulator lane: proxy row (1) / key (2)
+    const float alpha = P.alpha;
+    int buf = 0;
+    uint32_t bphase = 0;
+    for (int u = u_begin; u < u_end; ++u) {
+      const Unit x = decode(P, S, u);
+      const ReqInfo R = P.req[x.b];
+      float m_run = -INFINITY, z_run = 0.f;  // softmax pass state of this thread's row
+      Block blk{};
+      const float* cv = nullptr;
+      if (PASS == 2) {
+        blk = mass_block(P, S, x.tile);
+        cv = bf.cvals + (((size_t)x.l * P.B + x.b) * P.Hkv + x.h) * P.Prows_pad + blk.row0;
+      }
+      bool ok = true;
+      for (int kt = x.t0; kt < x.t1; kt += BK) {
+        if (!mbar_wait(&tfull[buf], bphase, abort_)) { ok = false; break; }
+        fence_after();
+        const uint32_t tacc = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * ACC_STRIDE);
+        if (PASS == 1) {
+          const int nvalid = min(BK, x.t1 - kt);
+          const uint32_t tcol = tacc + (uint32_t)(wg * 128);
+#pragma unroll 1
+          for (int c0 = 0; c0 < BK; c0 += 32) {
+            float v[32];
+            float (&v0)[16] = *reinterpret_cast<float(*)[16]>(v);
+            float (&v1)[16] = *reinterpret_cast<float(*)[16]>(v + 16);
+            tmem_ld16(tcol + c0, v0);
+            tmem_ld16(tcol + c0 + 16, v1);
+            tmem_wait_ld();
+            if (nvalid < c0 + 32) {
+#pragma unroll
+              for (int j = 0; j < 32; ++j)
+                if (c0 + j >= nvalid) v[j] = -INFINITY;
+            }
+            const float nm = -m_run;
+            float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+            for (int j = 0; j < 32; j += 4) {
+              s0 += fast_exp2(fmaf(v[j], alpha, nm));
+              s1 += fast_exp2(fmaf(v[j + 1], alpha, nm));
+              s2 += fast_exp2(fmaf(v[j + 2], alpha, nm));
+              s3 += fast_exp2(fmaf(v[j + 3], alpha, nm));
+            }
+            float zc = (s0 + s1) + (s2 + s3);
+            if (!(zc <= 1.8446744e19f)) {  // first chunk, overflow risk or NaN: raise the max
+              float cm = -INFINITY;
+#pragma unroll
+              for (int j = 0; j < 32; ++j) cm = fmaxf(cm, v[j] * alpha);
+              const float mn = fmaxf(m_run, cm);
+              if (mn == -INFINITY) {
+                zc = 0.f;
+              } else {
+                z_run *= fast_exp2(m_run - mn);
+                m_run = mn;
+                s0 = s1 = s2 = s3 = 0.f;
+#pragma unroll
+                for (int j = 0; j < 32; j += 4) {
+                  s0 += fast_exp2(fmaf(v[j], alpha, -mn));
+                  s1 += fast_exp2(fmaf(v[j + 1], alpha, -mn));
+                  s2 += fast_exp2(fmaf(v[j + 2], alpha, -mn));
+                  s3 += fast_exp2(fmaf(v[j + 3], alpha, -mn));
+                }
+                zc = (s0 + s1) + (s2 + s3);
+              }
+            }
+            z_run += zc;
+          }
+        } else {
+          const int t = kt + lrow;
+          const bool valid = t < x.t1;
+          const size_t col = (size_t)R.tok_off + t;
+          const int ng0 = (blk.ng + 1) / 2;
+          const int gb = wg == 0 ? 0 : ng0, ge = wg == 0 ? ng0 : blk.ng;
+          for (int gi = gb; gi < ge; ++gi) {
+            const float s = group_sum(tacc + (uint32_t)(gi * P.RG), cv + gi * P.RG, P.RG, alpha);
+            if (valid)
+              bf.gmass[(((size_t)x.l * P.Hkv + x.h) * P.G + blk.g0 + gi) * P.total_T + col] = s;
+          }
+          const bool my_anchor = blk.anchor && (blk.ng == 0 ? wg == 0 : wg == 1);
+          if (my_anchor) {
+            const int a0 = blk.ng * P.RG;
+            const float s = group_sum(tacc + (uint32_t)a0, cv + a0, P.anchor_rows, alpha);
+            if (valid)
+              bf.anchor[((size_t)x.l * P.Hkv + x.h) * P.total_T + col] = s / (float)P.r;
+          }
+        }
+        fence_before();
+        mbar_arrive(&tempty[buf]);
+        buf ^= 1;
+        if (buf == 0) bphase ^= 1u;
+      }
+      if (!ok) break;
+      if (PASS == 1) {
+        const int prow = x.tile * SROWS + wg * 128 + lrow;
+        bf.part[(((size_t)x.l * P.Hkv + x.h) * P.total_splits + R.split_off + x.split) *
+                    P.Prows_pad + prow] = make_float2(m_run, z_run);
+      }
+    }
+  }
+
+  fence_before();
+  __syncthreads();
+  if (warp == 1) tmem_dealloc(tmem, TMEM_COLS);
+  if (threadIdx.x == 0 && abort_flag) set_status(bf.status, kStatusTimeout);
+}
+
+// ---------------------------------------------------------------- host side
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static std::once_flag once;
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+bool make_map_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
+                 uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t box1) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[3] = {d0, d1, d2};
+  const cuuint64_t strides[2] = {stride1_bytes, stride2_bytes};
+  const cuuint32_t box[3] = {64, box1, 1};
+  const cuuint32_t es[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+Sched make_sched(const Problem& P, int pass) {
+  Sched s;
+  memset(&s, 0, sizeof(s));
+  if (pass == 1) {
+    s.ntiles = P.Prows_pad / SROWS;
+  } else {
+    s.gpt = P.G ? SROWS / P.RG : 1;
+    s.n_reg = P.G ? (P.G + s.gpt - 1) / s.gpt : 0;
+    const int last_rows = P.G ? (P.G - (s.n_reg - 1) * s.gpt) * P.RG : 0;
+    s.anchor_merged = (s.n_reg > 0 && last_rows + P.anchor_rows <= SROWS) ? 1 : 0;
+    s.ntiles = s.n_reg + (s.anchor_merged ? 0 : 1);
+  }
+  int acc = 0;
+  for (int b = 0; b < P.B; ++b) {
+    s.uoff[b] = acc;
+    acc += P.Hkv * s.ntiles * P.req[b].nsplit;
+  }
+  s.uoff[P.B] = acc;
+  s.units = acc * P.L;
+  return s;
+}
+
+int sm_count() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  return n;
+}
+
+template <int D>
+cudaError_t launch_d(const Problem& P, const Buffers& bf, cudaStream_t st, const void* K,
+                     cudaEvent_t* ev) {
+  using SM = Smem<D>;
+  CUtensorMap kmap, pmap;
+  const uint64_t ls = P.L > 1 ? (uint64_t)P.ls_kv : (uint64_t)P.total_T * P.Hkv * D;
+  if (!make_map_3d(&kmap, K, (uint64_t)P.Hkv * D, (uint64_t)P.total_T, (uint64_t)P.L,
+                   (uint64_t)P.Hkv * D * 2, ls * 2, BK))
+    return cudaErrorInvalidValue;
+  if (!make_map_3d(&pmap, bf.packed, D, (uint64_t)P.Prows_pad, (uint64_t)P.L * P.B * P.Hkv,
+                   (uint64_t)D * 2, (uint64_t)P.Prows_pad * D * 2, 16))
+    return cudaErrorInvalidValue;
+  const int nsm = sm_count();
+  if (nsm <= 0) return cudaErrorInvalidDevice;
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(score_umma_kernel<1, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                SM::DYN_BYTES)) != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(score_umma_kernel<2, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                SM::DYN_BYTES)) != cudaSuccess) return e;
+  const Sched s1 = make_sched(P, 1), s2 = make_sched(P, 2);
+  if (ev && (e = cudaEventRecord(ev[1], st)) != cudaSuccess) return e;
+  if (s1.units) {
+    score_umma_kernel<1, D><<<std::min(nsm, s1.units), NTHREADS, SM::DYN_BYTES, st>>>(kmap, pmap, P,
+                                                                                      s1, bf);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  if (ev && (e = cudaEventRecord(ev[2], st)) != cudaSuccess) return e;
+  if ((e = launch_merge(P, bf, st)) != cudaSuccess) return e;
+  if (ev && (e = cudaEventRecord(ev[3], st)) != cudaSuccess) return e;
+  if (s2.units) {
+    score_umma_kernel<2, D><<<std::min(nsm, s2.units), NTHREADS, SM::DYN_BYTES, st>>>(kmap, pmap, P,
+                                                                                      s2, bf);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+}  // namespace
+
+bool umma_supported(const Problem& P) {
+  if (P.dtype != MMSHIFT_BF16 || (P.d != 64 && P.d != 128)) return false;
+  if (P.RG > SROWS || P.anchor_rows > SROWS || P.Prows_pad % SROWS) return false;
+  if (P.L > 1 && (P.ls_kv % 8)) return false;   // TMA strides: multiples of 16 bytes
+  int dev = 0, major = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess)
+    return false;
+  return major == 10 && encode_fn() != nullptr;
+}
+
 int umma_launches(const Problem& P) { (void)P; return 3; }
 
 cudaError_t launch_score_umma(const Problem& P, const Buffers& bf, cudaStream_t st,
                               const void* K, cudaEvent_t* ev) {
-  (void)P; (void)bf; (void)st; (void)K; (void)ev;
-  return cudaErrorNotSupported;
+  if (reinterpret_cast<uintptr_t>(K) & 15) return cudaErrorMisalignedAddress;
+  return P.d == 128 ? launch_d<128>(P, bf, st, K, ev) : launch_d<64>(P, bf, st, K, ev);
 }
 
 }  // namespace mmshift

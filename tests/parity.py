@@ -107,7 +107,8 @@ def gpu_select(wl: S.Workload, layers, h, proxies=None):
     M.check(st, "mmshift_select")
     M.check(M.mmshift_poll_status(ws), "mmshift_poll_status")
     torch.cuda.synchronize()
-    return dict(idx=host(out_idx), out_k=host(out_k), out_v=host(out_v), group_mass=host(gm),
+    return dict(score_path=dbg.score_path, launches=dbg.launches,
+                idx=host(out_idx), out_k=host(out_k), out_v=host(out_v), group_mass=host(gm),
                 anchor=host(an), mass=host(ms), scores=host(sc), proxies=host(px),
                 K=np.stack([li.K for li in layers]), V=np.stack([li.V for li in layers]))
 

@@ -80,6 +80,8 @@ def test_select_given_proxies(name, mode):
     h = PT.hyper(score_mode=mode)
     prox = S.make_proxies(wl, h["n_proxies"], 0)
     gpu = PT.gpu_select(wl, [li], h, proxies=prox[None])
+    # bf16 scoring runs on the tensor cores, fp32 on the CUDA cores
+    assert gpu["score_path"] == (1 if wl.dtype == S.BF16 else 0)
     refs = PT.oracle_layer(wl, li, h, 0, proxies=prox)
     _check_all(wl, gpu, refs, h, what=name)
 
