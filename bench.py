@@ -397,6 +397,8 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="qwen7b-28l-32k", choices=sorted(S.WORKLOADS))
+    ap.add_argument("--layers", type=int, default=0,
+                    help="use only the first N layers of the workload (profiling runs)")
     ap.add_argument("--proxies", choices=["paper", "few"], default="paper",
                     help="paper: N=512, G=32 (Section 4.1); few: N=W, G=W/16")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
@@ -408,6 +410,8 @@ def main(argv=None):
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     wl = S.WORKLOADS[args.workload]
+    if args.layers:
+        wl = wl.replace(name=f"{wl.name}[:{args.layers} layers]", n_layers=min(args.layers, wl.n_layers))
     if args.impl == "reference":
         return run_reference(args, wl)
     return run_gpu(args, wl)

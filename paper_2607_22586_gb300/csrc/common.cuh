@@ -48,6 +48,7 @@ struct Problem {
   float rope_theta;
   int32_t rope_off;
   int32_t use_umma;    // steps 2-4 on the tensor cores (set per call)
+  int32_t part_slots;  // softmax partials per (row, key split): 1 (CUDA cores) or 2
   ReqInfo req[MMSHIFT_MAX_BATCH];
 };
 
@@ -56,7 +57,7 @@ struct Problem {
 struct Buffers {
   int* status;
   void* packed;       // [L][B][Hkv][Prows_pad][d] proxies, group-major rows
-  float2* part;       // [L][Hkv][total_splits][Prows_pad] (max, sum) partials
+  float2* part;       // [L][Hkv][total_splits][part_slots][Prows_pad] (max, sum) partials
   float* cvals;       // [L][B][Hkv][Prows_pad] log2 normaliser of each row
   float* gmass;       // [L][Hkv][G][T]
   float* anchor;      // [L][Hkv][T]

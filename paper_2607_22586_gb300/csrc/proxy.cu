@@ -61,17 +61,33 @@ __device__ __forceinline__ void box_muller(uint64_t a, uint64_t c, float& z0, fl
 
 // Four standard normals for dims 4q..4q+3 of proxy i of query head hq.
 __device__ __forceinline__ void normals4(const Problem& P, int i, int q, int hq, int b,
-                                         int layer, float z[4]) {
+                                         int layer, float& z0, float& z1, float& z2, float& z3) {
   uint64_t c[4] = {(uint64_t)i * (uint64_t)(P.d / 4) + (uint64_t)q, (uint64_t)hq,
                    (uint64_t)b, (uint64_t)(int64_t)layer};
   philox4x64_10(c, P.seed, 0ull);
-  box_muller(c[0], c[1], z[0], z[1]);
-  box_muller(c[2], c[3], z[2], z[3]);
+  box_muller(c[0], c[1], z0, z1);
+  box_muller(c[2], c[3], z2, z3);
 }
+
+// Four consecutive values rounded to T, one vector store.
+__device__ __forceinline__ void store4(__nv_bfloat16* dst, float a, float b, float c, float d) {
+  __nv_bfloat162 lo = __floats2bfloat162_rn(a, b), hi = __floats2bfloat162_rn(c, d);
+  uint2 u;
+  u.x = *reinterpret_cast<uint32_t*>(&lo);
+  u.y = *reinterpret_cast<uint32_t*>(&hi);
+  *reinterpret_cast<uint2*>(dst) = u;
+}
+__device__ __forceinline__ void store4(float* dst, float a, float b, float c, float d) {
+  *reinterpret_cast<float4*>(dst) = make_float4(a, b, c, d);
+}
+
+// Proxies of one query head are spread over kProxyChunks CTAs.
+constexpr int kProxyChunks = 8;
 
 template <typename T, int D>
 __global__ void __launch_bounds__(256) proxy_pack_kernel(Problem P, Buffers bf, const T* qwin) {
-  const int hq = blockIdx.x, b = blockIdx.y, l = blockIdx.z;
+  const int hq = blockIdx.x / kProxyChunks, chunk = blockIdx.x % kProxyChunks;
+  const int b = blockIdx.y, l = blockIdx.z;
   const int h = hq / P.r, j = hq - h * P.r;
   __shared__ float mu[D], sg[D], rc[D / 2], rs[D / 2];
   const T* q = qwin + (size_t)l * P.ls_q + ((size_t)b * P.W * P.Hq + hq) * D;
@@ -109,7 +125,9 @@ __global__ void __launch_bounds__(256) proxy_pack_kernel(Problem P, Buffers bf, 
   const T* pin = bf.proxies_in ? (const T*)bf.proxies_in + user_off : nullptr;
   T* pout = bf.proxies_out ? (T*)bf.proxies_out + user_off : nullptr;
   constexpr int NQ8 = D / 8;  // threads per proxy: dims [4qq, 4qq+4) and [D/2+4qq, +4)
-  for (int e = threadIdx.x; e < P.Np * NQ8; e += blockDim.x) {
+  const int per = (P.Np + kProxyChunks - 1) / kProxyChunks;
+  const int i0 = chunk * per, i1 = min(P.Np, i0 + per);
+  for (int e = i0 * NQ8 + threadIdx.x; e < i1 * NQ8; e += blockDim.x) {
     const int i = e / NQ8, qq = e - i * NQ8;
     float v[8];
     if (pin) {
@@ -120,8 +138,8 @@ __global__ void __launch_bounds__(256) proxy_pack_kernel(Problem P, Buffers bf, 
       }
     } else {
       float z[8];
-      normals4(P, i, qq, hq, b, layer, z);
-      normals4(P, i, qq + NQ8, hq, b, layer, z + 4);
+      normals4(P, i, qq, hq, b, layer, z[0], z[1], z[2], z[3]);
+      normals4(P, i, qq + NQ8, hq, b, layer, z[4], z[5], z[6], z[7]);
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
         const int d0 = 4 * qq + k, d1 = D / 2 + 4 * qq + k;
@@ -139,21 +157,17 @@ __global__ void __launch_bounds__(256) proxy_pack_kernel(Problem P, Buffers bf, 
       }
     }
     const int g = i / P.gs, ii = i - g * P.gs;
-    T* dst = packed ? packed + ((size_t)g * P.RG + (size_t)j * P.gs + ii) * D : nullptr;
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const T lo = from_f32<T>(v[k]), hi = from_f32<T>(v[4 + k]);
-      if (dst) {
-        dst[4 * qq + k] = lo;
-        dst[D / 2 + 4 * qq + k] = hi;
-      }
-      if (pout) {
-        pout[(size_t)i * D + 4 * qq + k] = lo;
-        pout[(size_t)i * D + D / 2 + 4 * qq + k] = hi;
-      }
+    if (packed) {
+      T* dst = packed + ((size_t)g * P.RG + (size_t)j * P.gs + ii) * D;
+      store4(dst + 4 * qq, v[0], v[1], v[2], v[3]);
+      store4(dst + D / 2 + 4 * qq, v[4], v[5], v[6], v[7]);
+    }
+    if (pout) {
+      store4(pout + (size_t)i * D + 4 * qq, v[0], v[1], v[2], v[3]);
+      store4(pout + (size_t)i * D + D / 2 + 4 * qq, v[4], v[5], v[6], v[7]);
     }
   }
-  if (!packed) return;
+  if (!packed || chunk != 0) return;
   // anchor row of this query head: the last window query as given
   T* arow = packed + (size_t)(P.n_group_rows + j) * D;
   for (int k = threadIdx.x; k < D; k += blockDim.x) arow[k] = q[(size_t)(P.W - 1) * qstride + k];
@@ -168,7 +182,7 @@ __global__ void __launch_bounds__(256) proxy_pack_kernel(Problem P, Buffers bf, 
 
 template <typename T, int D>
 cudaError_t launch_t(const Problem& P, const Buffers& bf, cudaStream_t st, const void* qwin) {
-  dim3 grid(P.Hq, P.B, P.L);
+  dim3 grid(P.Hq * kProxyChunks, P.B, P.L);
   proxy_pack_kernel<T, D><<<grid, 256, 0, st>>>(P, bf, (const T*)qwin);
   return cudaGetLastError();
 }

@@ -8,7 +8,8 @@
 //   the keys of its split through shared memory and keeps, per proxy row, an
 //   online (max, sum of exp2) pair of the log2-scaled logits x = s * alpha,
 //   alpha = softmax_scale * log2(e).
-// Merge: combines the splits of each row into c = m + log2(Z) (the log2
+// Merge: combines the partials of each row (one per key split, two on the
+//   tensor-core path) in a fixed order into c = m + log2(Z) (the log2
 //   normaliser), +inf for padding rows so they weigh nothing.
 // Pass 2: CTA = (layer, KV head, 64 keys). It streams every packed proxy row,
 //   recomputes the logits and adds exp2(x - c) into per-(group, key) sums in a
@@ -113,8 +114,8 @@ __global__ void __launch_bounds__(256) pass1_simt(Problem P, Buffers bf, const T
     merge_ms(run_m, run_z, m, z);
   }
   if (part == 0)
-    bf.part[(((size_t)l * P.Hkv + h) * P.total_splits + s) * P.Prows_pad + rt * TILE + row] =
-        make_float2(run_m, run_z);
+    bf.part[(((size_t)l * P.Hkv + h) * P.total_splits + s) * P.part_slots * P.Prows_pad +
+            rt * TILE + row] = make_float2(run_m, run_z);
 }
 
 __global__ void merge_kernel(Problem P, Buffers bf) {
@@ -124,8 +125,9 @@ __global__ void merge_kernel(Problem P, Buffers bf) {
   if (p >= P.Prows_pad) return;
   const ReqInfo R = P.req[b];
   float m = -INFINITY, z = 0.f;
-  const float2* src = bf.part + (((size_t)l * P.Hkv + h) * P.total_splits + R.split_off) * P.Prows_pad + p;
-  for (int s = 0; s < R.nsplit; ++s) {
+  const float2* src =
+      bf.part + (((size_t)l * P.Hkv + h) * P.total_splits + R.split_off) * P.part_slots * P.Prows_pad + p;
+  for (int s = 0; s < R.nsplit * P.part_slots; ++s) {
     const float2 v = src[(size_t)s * P.Prows_pad];
     merge_ms(m, z, v.x, v.y);
   }

@@ -8,12 +8,15 @@
 //               the work unit changes) and a 4-stage ring of 128-key K tiles;
 //   warp 1      TMEM allocator and MMA issuer (one thread): d/16 tcgen05.mma
 //               of K = 16 per key tile into one of two TMEM accumulators;
-//   warps 2-9   epilogue (two warpgroups): tcgen05.ld of the accumulator,
-//               exp2 and reductions in registers, outputs to global memory.
-// Work units are (layer, request, KV head, proxy block, key split of 1024
-// keys), split fastest; each CTA takes a contiguous range of units, so the
-// stationary block changes rarely and the split boundaries (and so the
-// merge order of the softmax partials) are those of the CUDA-core path.
+//   warps 2-17  epilogue (four warpgroups, two per TMEM accumulator):
+//               tcgen05.ld of the accumulator, exp2 and reductions in
+//               registers, outputs to global memory.
+// Work units are (layer, request, KV head, key split of 1024 keys, proxy
+// block). Teams of one CTA per proxy block walk contiguous ranges of key
+// splits, so the team's CTAs read each K tile together (DRAM once, then L2)
+// and a CTA's stationary block changes only with the (layer, request, head).
+// The split boundaries (and so the merge order of the softmax partials) are
+// those of the CUDA-core path.
 //
 // Softmax pass (PASS 1): stationary = 2 x 128 proxy rows as the M operand,
 //   K tile = N operand (M=128, N=128, two MMAs); the accumulator lane is a
@@ -43,9 +46,9 @@ using namespace umma;
 constexpr int BK = 128;          // keys per K tile
 constexpr int SROWS = 256;       // stationary proxy rows per block
 constexpr int NSTAGE = 4;        // K-tile ring depth
-constexpr int NTHREADS = 320;
+constexpr int NTHREADS = 576;
 constexpr int EPI_WARP0 = 2;
-constexpr int NEPI = 256;        // epilogue threads
+constexpr int NEPI = 512;        // epilogue threads: 4 warpgroups, 2 per accumulator
 constexpr int TMEM_COLS = 512;
 constexpr int ACC_STRIDE = 256;  // TMEM columns per accumulator buffer
 
@@ -72,10 +75,10 @@ __device__ __forceinline__ Unit decode(const Problem& P, const Sched& S, int u) 
   x.b = b;
   r -= S.uoff[b];
   const int ns = P.req[b].nsplit;
-  x.split = r % ns;
-  r /= ns;
   x.tile = r % S.ntiles;
-  x.h = r / S.ntiles;
+  r /= S.ntiles;
+  x.split = r % ns;
+  x.h = r / ns;
   x.t0 = x.split * P.split_len;
   x.t1 = min(P.req[b].t_len, x.t0 + P.split_len);
   return x;
@@ -118,31 +121,91 @@ struct Smem {
   static constexpr int DYN_BYTES = 1024 + STAT_BYTES + RING_BYTES;
 };
 
-// Sum over the RG (multiple of 16) accumulator columns of one group:
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  tmem_ld16(taddr, *reinterpret_cast<float(*)[16]>(v));
+  tmem_ld16(taddr + 16, *reinterpret_cast<float(*)[16]>(v + 16));
+}
+
+// Online (max, sum of exp2) update of one row over 32 logits v (columns
+// c0..c0+31 of the tile; columns >= nvalid are past the split and ignored).
+// m is the running max of the log2-scaled logits, z the sum of exp2(x - m).
+// The max is only raised when the chunk's sum relative to it would exceed
+// 2^64 (or on the first chunk), so the common path is FFMA + EX2 + FADD.
+__device__ __forceinline__ void softmax_chunk(float (&v)[32], int c0, int nvalid, float alpha,
+                                              float& m, float& z) {
+  if (nvalid < c0 + 32) {
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (c0 + j >= nvalid) v[j] = -INFINITY;
+  }
+  const float nm = -m;
+  float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+  for (int j = 0; j < 32; j += 4) {
+    s0 += fast_exp2(fmaf(v[j], alpha, nm));
+    s1 += fast_exp2(fmaf(v[j + 1], alpha, nm));
+    s2 += fast_exp2(fmaf(v[j + 2], alpha, nm));
+    s3 += fast_exp2(fmaf(v[j + 3], alpha, nm));
+  }
+  float zc = (s0 + s1) + (s2 + s3);
+  if (!(zc <= 1.8446744e19f)) {  // first chunk, overflow risk or NaN: raise the max
+    float cm = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) cm = fmaxf(cm, v[j] * alpha);
+    const float mn = fmaxf(m, cm);
+    if (mn == -INFINITY) {
+      zc = 0.f;
+    } else {
+      z *= fast_exp2(m - mn);
+      m = mn;
+      s0 = s1 = s2 = s3 = 0.f;
+#pragma unroll
+      for (int j = 0; j < 32; j += 4) {
+        s0 += fast_exp2(fmaf(v[j], alpha, -mn));
+        s1 += fast_exp2(fmaf(v[j + 1], alpha, -mn));
+        s2 += fast_exp2(fmaf(v[j + 2], alpha, -mn));
+        s3 += fast_exp2(fmaf(v[j + 3], alpha, -mn));
+      }
+      zc = (s0 + s1) + (s2 + s3);
+    }
+  }
+  z += zc;
+}
+
+__device__ __forceinline__ void load_c16(const float* __restrict__ c, float (&cv)[16]) {
+  const float4* c4 = reinterpret_cast<const float4*>(c);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float4 t = __ldg(c4 + i);
+    cv[4 * i] = t.x; cv[4 * i + 1] = t.y; cv[4 * i + 2] = t.z; cv[4 * i + 3] = t.w;
+  }
+}
+
+__device__ __forceinline__ void mass_chunk(const float (&v)[16], const float (&cv)[16],
+                                           float alpha, float (&a)[4]) {
+#pragma unroll
+  for (int j = 0; j < 16; j += 4) {
+    a[0] += fast_exp2(fmaf(v[j], alpha, -cv[j]));
+    a[1] += fast_exp2(fmaf(v[j + 1], alpha, -cv[j + 1]));
+    a[2] += fast_exp2(fmaf(v[j + 2], alpha, -cv[j + 2]));
+    a[3] += fast_exp2(fmaf(v[j + 3], alpha, -cv[j + 3]));
+  }
+}
+
+// Sum over the ncols (multiple of 16) accumulator columns of one group:
 // sum_j exp2(acc_j * alpha - c_j), four partial sums added in a fixed order.
 __device__ __forceinline__ float group_sum(uint32_t tcol, const float* __restrict__ c, int ncols,
                                            float alpha) {
-  float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+  float a[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 1
   for (int cc = 0; cc < ncols; cc += 16) {
-    float v[16];
+    float v[16], cv[16];
     tmem_ld16(tcol + cc, v);
-    const float4* c4 = reinterpret_cast<const float4*>(c + cc);
-    float cv[16];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const float4 t = __ldg(c4 + i);
-      cv[4 * i] = t.x; cv[4 * i + 1] = t.y; cv[4 * i + 2] = t.z; cv[4 * i + 3] = t.w;
-    }
+    load_c16(c + cc, cv);
     tmem_wait_ld();
-#pragma unroll
-    for (int j = 0; j < 16; j += 4) {
-      a0 += fast_exp2(fmaf(v[j], alpha, -cv[j]));
-      a1 += fast_exp2(fmaf(v[j + 1], alpha, -cv[j + 1]));
-      a2 += fast_exp2(fmaf(v[j + 2], alpha, -cv[j + 2]));
-      a3 += fast_exp2(fmaf(v[j + 3], alpha, -cv[j + 3]));
-    }
+    mass_chunk(v, cv, alpha, a);
   }
-  return (a0 + a1) + (a2 + a3);
+  return (a[0] + a[1]) + (a[2] + a[3]);
 }
 
 template <int PASS, int D>
@@ -162,8 +225,17 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   volatile int* abort_ = &abort_flag;
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int u_begin = (int)((long long)blockIdx.x * S.units / gridDim.x);
-  const int u_end = (int)((long long)(blockIdx.x + 1) * S.units / gridDim.x);
+  // Team schedule: the grid is a multiple of the stationary blocks per
+  // (request, KV head); team j = CTAs [j*ntiles, (j+1)*ntiles), one per block.
+  // A team walks a contiguous range of key splits (over layers, requests and
+  // heads); all its CTAs read the same split at the same time, so each K tile
+  // comes from DRAM once and from L2 for the others, and a CTA reloads its
+  // stationary block only when the (layer, request, head) changes.
+  const int nteams = gridDim.x / S.ntiles;
+  const int team = blockIdx.x / S.ntiles, my_tile = blockIdx.x % S.ntiles;
+  const int nsplit_rows = S.units / S.ntiles;
+  const int s_begin = (int)((long long)team * nsplit_rows / nteams);
+  const int s_end = (int)((long long)(team + 1) * nsplit_rows / nteams);
 
   if (threadIdx.x == 0) {
     abort_flag = 0;
@@ -175,7 +247,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     mbar_init(&sempty, 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(&tfull[i], 1);
-      mbar_init(&tempty[i], NEPI);
+      mbar_init(&tempty[i], NEPI / 2);
     }
     fence_barrier_init();
     prefetch_tmap(&kmap);
@@ -196,7 +268,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       int stage = 0;
       uint32_t phase = 0, sphase = 0;
       long long prev = -1;
-      for (int u = u_begin; u < u_end; ++u) {
+      for (int sr = s_begin; sr < s_end; ++sr) {
+        const int u = sr * S.ntiles + my_tile;
         const Unit x = decode(P, S, u);
         const long long key = block_key(P, S, x);
         if (key != prev) {
@@ -238,7 +311,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       uint32_t phase = 0, bphase = 0, sphase = 0;
       long long prev = -1;
       uint32_t idesc = idesc_bf16_f32(128, 128);
-      for (int u = u_begin; u < u_end; ++u) {
+      for (int sr = s_begin; sr < s_end; ++sr) {
+        const int u = sr * S.ntiles + my_tile;
         const Unit x = decode(P, S, u);
         const long long key = block_key(P, S, x);
         if (key != prev) {
@@ -283,14 +357,19 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    const int ew = warp - EPI_WARP0;      // 0..7
-    const int wg = ew / 4;                // warpgroup
+    // Warpgroups 0,1 drain accumulator 0, warpgroups 2,3 accumulator 1, so
+    // each warpgroup takes every other key tile. In the softmax pass the
+    // two warpgroups of a pair own the two 128-row M tiles; in the mass pass
+    // they split the groups of the stationary block.
+    const int ew = warp - EPI_WARP0;      // 0..15
+    const int wg = ew / 4;                // warpgroup 0..3
+    const int par = wg >> 1, sub = wg & 1;
     const int q = warp % 4;               // TMEM lane quarter this warp may access
     const int lrow = q * 32 + lane;       // accumulator lane: proxy row (1) / key (2)
     const float alpha = P.alpha;
-    int buf = 0;
-    uint32_t bphase = 0;
-    for (int u = u_begin; u < u_end; ++u) {
+    uint32_t ntile = 0;                   // tiles seen, in the MMA's order
+    for (int sr = s_begin; sr < s_end; ++sr) {
+      const int u = sr * S.ntiles + my_tile;
       const Unit x = decode(P, S, u);
       const ReqInfo R = P.req[x.b];
       float m_run = -INFINITY, z_run = 0.f;  // softmax pass state of this thread's row
@@ -301,87 +380,48 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         cv = bf.cvals + (((size_t)x.l * P.B + x.b) * P.Hkv + x.h) * P.Prows_pad + blk.row0;
       }
       bool ok = true;
-      for (int kt = x.t0; kt < x.t1; kt += BK) {
-        if (!mbar_wait(&tfull[buf], bphase, abort_)) { ok = false; break; }
+      for (int kt = x.t0; kt < x.t1; kt += BK, ++ntile) {
+        const int buf = (int)(ntile & 1u);
+        if (buf != par) continue;
+        if (!mbar_wait(&tfull[buf], (ntile >> 1) & 1u, abort_)) { ok = false; break; }
         fence_after();
         const uint32_t tacc = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * ACC_STRIDE);
         if (PASS == 1) {
           const int nvalid = min(BK, x.t1 - kt);
-          const uint32_t tcol = tacc + (uint32_t)(wg * 128);
+          const uint32_t tcol = tacc + (uint32_t)(sub * 128);
 #pragma unroll 1
           for (int c0 = 0; c0 < BK; c0 += 32) {
             float v[32];
-            float (&v0)[16] = *reinterpret_cast<float(*)[16]>(v);
-            float (&v1)[16] = *reinterpret_cast<float(*)[16]>(v + 16);
-            tmem_ld16(tcol + c0, v0);
-            tmem_ld16(tcol + c0 + 16, v1);
+            tmem_ld32(tcol + c0, v);
             tmem_wait_ld();
-            if (nvalid < c0 + 32) {
-#pragma unroll
-              for (int j = 0; j < 32; ++j)
-                if (c0 + j >= nvalid) v[j] = -INFINITY;
-            }
-            const float nm = -m_run;
-            float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-#pragma unroll
-            for (int j = 0; j < 32; j += 4) {
-              s0 += fast_exp2(fmaf(v[j], alpha, nm));
-              s1 += fast_exp2(fmaf(v[j + 1], alpha, nm));
-              s2 += fast_exp2(fmaf(v[j + 2], alpha, nm));
-              s3 += fast_exp2(fmaf(v[j + 3], alpha, nm));
-            }
-            float zc = (s0 + s1) + (s2 + s3);
-            if (!(zc <= 1.8446744e19f)) {  // first chunk, overflow risk or NaN: raise the max
-              float cm = -INFINITY;
-#pragma unroll
-              for (int j = 0; j < 32; ++j) cm = fmaxf(cm, v[j] * alpha);
-              const float mn = fmaxf(m_run, cm);
-              if (mn == -INFINITY) {
-                zc = 0.f;
-              } else {
-                z_run *= fast_exp2(m_run - mn);
-                m_run = mn;
-                s0 = s1 = s2 = s3 = 0.f;
-#pragma unroll
-                for (int j = 0; j < 32; j += 4) {
-                  s0 += fast_exp2(fmaf(v[j], alpha, -mn));
-                  s1 += fast_exp2(fmaf(v[j + 1], alpha, -mn));
-                  s2 += fast_exp2(fmaf(v[j + 2], alpha, -mn));
-                  s3 += fast_exp2(fmaf(v[j + 3], alpha, -mn));
-                }
-                zc = (s0 + s1) + (s2 + s3);
-              }
-            }
-            z_run += zc;
+            softmax_chunk(v, c0, nvalid, alpha, m_run, z_run);
           }
         } else {
           const int t = kt + lrow;
           const bool valid = t < x.t1;
           const size_t col = (size_t)R.tok_off + t;
           const int ng0 = (blk.ng + 1) / 2;
-          const int gb = wg == 0 ? 0 : ng0, ge = wg == 0 ? ng0 : blk.ng;
+          const int gb = sub == 0 ? 0 : ng0, ge = sub == 0 ? ng0 : blk.ng;
           for (int gi = gb; gi < ge; ++gi) {
-            const float s = group_sum(tacc + (uint32_t)(gi * P.RG), cv + gi * P.RG, P.RG, alpha);
+            const float sm = group_sum(tacc + (uint32_t)(gi * P.RG), cv + gi * P.RG, P.RG, alpha);
             if (valid)
-              bf.gmass[(((size_t)x.l * P.Hkv + x.h) * P.G + blk.g0 + gi) * P.total_T + col] = s;
+              bf.gmass[(((size_t)x.l * P.Hkv + x.h) * P.G + blk.g0 + gi) * P.total_T + col] = sm;
           }
-          const bool my_anchor = blk.anchor && (blk.ng == 0 ? wg == 0 : wg == 1);
+          const bool my_anchor = blk.anchor && (blk.ng == 0 ? sub == 0 : sub == 1);
           if (my_anchor) {
             const int a0 = blk.ng * P.RG;
-            const float s = group_sum(tacc + (uint32_t)a0, cv + a0, P.anchor_rows, alpha);
+            const float sm = group_sum(tacc + (uint32_t)a0, cv + a0, P.anchor_rows, alpha);
             if (valid)
-              bf.anchor[((size_t)x.l * P.Hkv + x.h) * P.total_T + col] = s / (float)P.r;
+              bf.anchor[((size_t)x.l * P.Hkv + x.h) * P.total_T + col] = sm / (float)P.r;
           }
         }
         fence_before();
         mbar_arrive(&tempty[buf]);
-        buf ^= 1;
-        if (buf == 0) bphase ^= 1u;
       }
       if (!ok) break;
       if (PASS == 1) {
-        const int prow = x.tile * SROWS + wg * 128 + lrow;
-        bf.part[(((size_t)x.l * P.Hkv + x.h) * P.total_splits + R.split_off + x.split) *
+        const int prow = x.tile * SROWS + sub * 128 + lrow;
+        bf.part[((((size_t)x.l * P.Hkv + x.h) * P.total_splits + R.split_off + x.split) * 2 + par) *
                     P.Prows_pad + prow] = make_float2(m_run, z_run);
       }
     }
@@ -470,9 +510,16 @@ cudaError_t launch_d(const Problem& P, const Buffers& bf, cudaStream_t st, const
   if ((e = cudaFuncSetAttribute(score_umma_kernel<2, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 SM::DYN_BYTES)) != cudaSuccess) return e;
   const Sched s1 = make_sched(P, 1), s2 = make_sched(P, 2);
+  // whole teams of ntiles CTAs (one per stationary block), at most one CTA
+  // per SM while the work allows
+  auto grid_of = [nsm](const Sched& s) {
+    const int rows = s.units / s.ntiles;
+    const int nteams = std::max(1, std::min(nsm / s.ntiles, rows));
+    return nteams * s.ntiles;
+  };
   if (ev && (e = cudaEventRecord(ev[1], st)) != cudaSuccess) return e;
   if (s1.units) {
-    score_umma_kernel<1, D><<<std::min(nsm, s1.units), NTHREADS, SM::DYN_BYTES, st>>>(kmap, pmap, P,
+    score_umma_kernel<1, D><<<grid_of(s1), NTHREADS, SM::DYN_BYTES, st>>>(kmap, pmap, P,
                                                                                       s1, bf);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
@@ -480,7 +527,7 @@ cudaError_t launch_d(const Problem& P, const Buffers& bf, cudaStream_t st, const
   if ((e = launch_merge(P, bf, st)) != cudaSuccess) return e;
   if (ev && (e = cudaEventRecord(ev[3], st)) != cudaSuccess) return e;
   if (s2.units) {
-    score_umma_kernel<2, D><<<std::min(nsm, s2.units), NTHREADS, SM::DYN_BYTES, st>>>(kmap, pmap, P,
+    score_umma_kernel<2, D><<<grid_of(s2), NTHREADS, SM::DYN_BYTES, st>>>(kmap, pmap, P,
                                                                                       s2, bf);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }

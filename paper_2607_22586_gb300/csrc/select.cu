@@ -3,29 +3,33 @@
 // (Appendix B).
 //
 // Both selections are radix selects on order-preserving 32-bit keys of the
-// float values, 8 bits per pass from the top, with warp-aggregated histogram
-// updates (__match_any_sync groups lanes with the same digit; the group leader
-// adds the group's count, and its weight summed with __reduce_add_sync). No
-// full sort is done.
+// non-negative float values -- no full sort. Digits: the 8 exponent bits, then
+// 8, 8 and 7 mantissa bits. Each warp owns a private 256-bin histogram in
+// shared memory (counts, and for the weighted select a 64-bit fixed-point
+// weight kept as two 32-bit words whose carry is detected from the atomic's
+// return value), so atomics only contend inside a warp; after the first digit
+// only the few keys matching the prefix are counted and warps without any skip
+// the pass.
 //  - cover_kernel: one CTA per (layer, request, KV head, group). Weighted
 //    select: the smallest prefix of keys in (mass desc, t asc) order whose
 //    mass reaches tau * total. Masses are summed in 64-bit fixed point (2^-S
-//    units, S <= 40, chosen per group so the total cannot overflow), so the
-//    sums are exact and order-independent. Output: the cover set as a bitmap
-//    (one bit per key).
+//    units, S <= 40, chosen per group so the total cannot overflow), so sums
+//    are exact and order-independent. Output: the cover set as a bitmap.
 //  - topk_kernel: one CTA per (layer, request, KV head). Builds S_t (votes
-//    from the bitmaps plus lambda * anchor, or the summed mass), then a count
-//    select of the C-1 largest among t < T-1 (ties: lower t), and an ordered
-//    compaction with warp ballots that writes the kept indices ascending with
-//    T-1 last.
+//    counted from the bitmaps with warp ballots, plus lambda * anchor; or the
+//    summed mass), then a count select of the C-1 largest among t < T-1
+//    (ties: lower t) and an ordered compaction with warp ballots that writes
+//    the kept indices ascending with T-1 last.
 #include "common.cuh"
 
 namespace mmshift {
 namespace {
 
-constexpr int NT = 1024;          // threads per selection CTA
+constexpr int NT = 512;           // threads per selection CTA
 constexpr int NW = NT / 32;
-constexpr int kMaxStaged = 49152; // keys staged in shared memory (192 KB)
+constexpr int NBIN = 256;
+constexpr int kMaxStaged = 40960; // keys staged in shared memory (160 KB)
+constexpr int HIST_WORDS = 3 * NW * NBIN;  // per-warp count / weight-lo / weight-hi
 
 __device__ __forceinline__ uint32_t ordered_key(float x) {
   uint32_t u = __float_as_uint(x + 0.0f);  // -0 -> +0
@@ -34,16 +38,20 @@ __device__ __forceinline__ uint32_t ordered_key(float x) {
 __device__ __forceinline__ float key_value(uint32_t k) {
   return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
 }
+// Keys of non-negative values (negatives and NaN are clamped to +0).
+__device__ __forceinline__ uint32_t nonneg_key(float x) {
+  return ordered_key(fmaxf(x, 0.f));
+}
 
 struct SelShared {
-  unsigned long long hw[256];
-  unsigned int hn[256];
+  unsigned long long total;
   unsigned long long wsum[NW];
   unsigned int wcnt[NW];
   unsigned long long cum_w;
   unsigned int cum_n;
   unsigned int digit;
   unsigned int prefix;
+  unsigned int n_theta;
   int aux;
   float fsum;
 };
@@ -53,7 +61,7 @@ struct KeySrc {
   const uint32_t* smem;
   const float* gmem;
   __device__ __forceinline__ uint32_t operator()(int i) const {
-    return smem ? smem[i] : ordered_key(gmem[i]);
+    return smem ? smem[i] : nonneg_key(gmem[i]);
   }
 };
 
@@ -74,47 +82,90 @@ __device__ __forceinline__ unsigned warp_excl_prefix(SelShared& S, unsigned mine
 }
 
 // Smallest prefix of the (key desc, index asc) order whose cumulative weight
-// is >= target_w and whose length is >= target_n. On return S.prefix is the
-// key theta of the prefix's last element, S.cum_w / S.cum_n the weight / count
-// of keys > theta, and the return value is the number of keys equal to theta.
+// is >= target_w and whose length is >= target_n (all keys >= 0x80000000,
+// i.e. of non-negative values). On return S.prefix is the key theta of the
+// prefix's last element, S.cum_w / S.cum_n the weight / count of keys above
+// theta and S.n_theta the number of keys equal to theta. `hist` is
+// HIST_WORDS words of shared memory.
+//
+// Weighted mode: target_w is derived from the exact fixed-point total, summed in
+// the first pass: target_w = min(total, ceil(tau * total)); S.total holds it.
 template <bool WEIGHTED>
-__device__ unsigned radix_select(const KeySrc& get, int n, unsigned long long target_w,
-                                 unsigned target_n, int shift, SelShared& S) {
-  const int tid = threadIdx.x, lane = tid & 31;
-  uint32_t prefix = 0, mask = 0;
+__device__ void radix_select(const KeySrc& get, int n, unsigned long long target_w,
+                             unsigned target_n, int shift, float tau, SelShared& S,
+                             uint32_t* hist) {
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  uint32_t* hn = hist + w * NBIN;
+  uint32_t* hlo = hist + (NW + w) * NBIN;
+  uint32_t* hhi = hist + (2 * NW + w) * NBIN;
   if (tid == 0) { S.cum_w = 0; S.cum_n = 0; }
-  unsigned n_theta = 0;
+  uint32_t prefix = 0x80000000u;
+  constexpr int kSh[4] = {23, 15, 7, 0};
+  constexpr int kWid[4] = {8, 8, 8, 7};
+#pragma unroll 1
   for (int pass = 0; pass < 4; ++pass) {
-    const int sh = 24 - 8 * pass;
-    for (int i = tid; i < 256; i += NT) { S.hw[i] = 0; S.hn[i] = 0; }
-    __syncthreads();
+    const int sh = kSh[pass], hs = sh + kWid[pass];
+    const uint32_t dmask = (1u << kWid[pass]) - 1u;
+    for (int i = lane; i < NBIN; i += 32) {
+      hn[i] = 0;
+      if (WEIGHTED) { hlo[i] = 0; hhi[i] = 0; }
+    }
+    __syncwarp();
+    unsigned long long tot = 0;
     for (int base = 0; base < n; base += NT) {
       const int i = base + tid;
       const uint32_t k = i < n ? get(i) : 0u;
-      const bool take = i < n && (k & mask) == prefix;
-      const unsigned dig = take ? ((k >> sh) & 255u) : 256u;
-      const unsigned peers = __match_any_sync(0xffffffffu, dig);
-      const bool leader = take && lane == (__ffs(peers) - 1);
-      if (WEIGHTED) {
-        const unsigned long long w = take ? fx_weight(k, shift) : 0ull;
-        const unsigned s0 = __reduce_add_sync(peers, (unsigned)(w & 0x1fffffull));
-        const unsigned s1 = __reduce_add_sync(peers, (unsigned)((w >> 21) & 0x1fffffull));
-        const unsigned s2 = __reduce_add_sync(peers, (unsigned)(w >> 42));
-        if (leader)
-          atomicAdd(&S.hw[dig], (unsigned long long)s0 + ((unsigned long long)s1 << 21) +
-                                    ((unsigned long long)s2 << 42));
+      const bool take = i < n && (k >> hs) == (prefix >> hs);
+      if (pass > 0 && !__any_sync(0xffffffffu, take)) continue;
+      if (take) {
+        const uint32_t d = (k >> sh) & dmask;
+        atomicAdd(&hn[d], 1u);
+        if (WEIGHTED) {
+          const unsigned long long wt = fx_weight(k, shift);
+          if (pass == 0) tot += wt;
+          const uint32_t lo = (uint32_t)wt;
+          uint32_t hi = (uint32_t)(wt >> 32);
+          if (lo) {
+            const uint32_t old = atomicAdd(&hlo[d], lo);
+            hi += (old + lo < old) ? 1u : 0u;   // carry out of the low word
+          }
+          if (hi) atomicAdd(&hhi[d], hi);
+        }
       }
-      if (leader) atomicAdd(&S.hn[dig], (unsigned)__popc(peers));
+    }
+    if (WEIGHTED && pass == 0) {
+      for (int off = 16; off; off >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, off);
+      if (lane == 0) S.wsum[w] = tot;
     }
     __syncthreads();
+    if (WEIGHTED && pass == 0) {
+      unsigned long long total = 0;
+      for (int i = 0; i < NW; ++i) total += S.wsum[i];
+      unsigned long long t = (unsigned long long)ceil((double)tau * (double)total);
+      target_w = t > total ? total : t;
+      if (tid == 0) S.total = total;
+    }
     if (tid < 32) {
       // lane L owns digits 255-8L .. 248-8L, scanned from the top
+      unsigned long long bw[8];
+      unsigned bn[8];
       unsigned long long sw = 0;
       unsigned sn = 0;
+#pragma unroll
       for (int k = 0; k < 8; ++k) {
         const int d = 255 - 8 * lane - k;
-        sw += S.hw[d];
-        sn += S.hn[d];
+        unsigned long long wsum = 0;
+        unsigned nsum = 0;
+        for (int ww = 0; ww < NW; ++ww) {
+          nsum += hist[ww * NBIN + d];
+          if (WEIGHTED)
+            wsum += (unsigned long long)hist[(NW + ww) * NBIN + d] +
+                    ((unsigned long long)hist[(2 * NW + ww) * NBIN + d] << 32);
+        }
+        bw[k] = wsum;
+        bn[k] = nsum;
+        sw += wsum;
+        sn += nsum;
       }
       unsigned long long iw = sw;
       unsigned in = sn;
@@ -131,33 +182,40 @@ __device__ unsigned radix_select(const KeySrc& get, int n, unsigned long long ta
       if (lane == f) {
         unsigned long long c_w = cw + iw - sw;
         unsigned c_n = cn + in - sn;
-        int chosen = 255 - 8 * lane - 7;
+        int chosen = 7;
+        unsigned n_ch = bn[7];
+        bool found = false;
+#pragma unroll
         for (int k = 0; k < 8; ++k) {
-          const int d = 255 - 8 * lane - k;
-          if ((!WEIGHTED || c_w + S.hw[d] >= target_w) && c_n + S.hn[d] >= target_n) {
-            chosen = d;
-            break;
+          if (!found) {
+            if ((!WEIGHTED || c_w + bw[k] >= target_w) && c_n + bn[k] >= target_n) {
+              chosen = k;
+              n_ch = bn[k];
+              found = true;
+            } else if (k < 7) {
+              c_w += bw[k];
+              c_n += bn[k];
+            }
           }
-          if (k < 7) { c_w += S.hw[d]; c_n += S.hn[d]; }
         }
         S.cum_w = c_w;
         S.cum_n = c_n;
-        S.digit = (unsigned)chosen;
+        S.digit = (unsigned)(255 - 8 * lane - chosen);
+        S.n_theta = n_ch;
       }
     }
     __syncthreads();
-    prefix |= S.digit << sh;
-    mask |= 255u << sh;
-    n_theta = S.hn[S.digit];
+    prefix |= (S.digit & dmask) << sh;
     __syncthreads();
   }
   if (tid == 0) S.prefix = prefix;
   __syncthreads();
-  return n_theta;
 }
 
-__global__ void __launch_bounds__(NT) cover_kernel(Problem P, Buffers bf) {
-  extern __shared__ uint32_t keys_sm[];
+__global__ void __launch_bounds__(NT, 1) cover_kernel(Problem P, Buffers bf) {
+  extern __shared__ uint32_t dyn[];
+  uint32_t* hist = dyn;
+  uint32_t* keys_sm = dyn + HIST_WORDS;
   __shared__ SelShared S;
   const int g = blockIdx.x % P.G, h = blockIdx.x / P.G, b = blockIdx.y, l = blockIdx.z;
   const ReqInfo R = P.req[b];
@@ -168,9 +226,9 @@ __global__ void __launch_bounds__(NT) cover_kernel(Problem P, Buffers bf) {
   // stage keys and sum the masses (float, only to choose the fixed point)
   float fs = 0.f;
   for (int i = tid; i < n; i += NT) {
-    const float x = m[i];
+    const float x = fmaxf(m[i], 0.f);
     if (staged) keys_sm[i] = ordered_key(x);
-    fs += fmaxf(x, 0.f);
+    fs += x;
   }
   for (int off = 16; off; off >>= 1) fs += __shfl_xor_sync(0xffffffffu, fs, off);
   if (lane == 0) S.wsum[w] = __float_as_uint(fs);
@@ -185,47 +243,40 @@ __global__ void __launch_bounds__(NT) cover_kernel(Problem P, Buffers bf) {
   frexpf(S.fsum + 1.0f, &e);               // S.fsum + 1 < 2^e
   const int shift = max(0, min(40, 60 - e));
   KeySrc get{staged ? keys_sm : nullptr, m};
-  // exact fixed-point total
-  unsigned long long tw = 0;
-  for (int i = tid; i < n; i += NT) tw += fx_weight(get(i), shift);
-  for (int off = 16; off; off >>= 1) tw += __shfl_xor_sync(0xffffffffu, tw, off);
-  __syncthreads();
-  if (lane == 0) S.wsum[w] = tw;
-  __syncthreads();
-  unsigned long long total = 0;
-  for (int i = 0; i < NW; ++i) total += S.wsum[i];
-  __syncthreads();
-  unsigned long long target = (unsigned long long)ceil((double)P.tau * (double)total);
-  if (target > total) target = total;
-  const unsigned n_theta = radix_select<true>(get, n, target, 1u, shift, S);
+  radix_select<true>(get, n, 0ull, 1u, shift, P.tau, S, hist);
   const uint32_t theta = S.prefix;
+  const unsigned n_theta = S.n_theta;
+  const unsigned long long target = min(S.total, (unsigned long long)ceil((double)P.tau * (double)S.total));
   const unsigned long long wth = fx_weight(theta, shift);
   const unsigned long long need_w = target > S.cum_w ? target - S.cum_w : 0ull;
   unsigned n_tie = 1;
   if (need_w > 0 && wth > 0) n_tie = (unsigned)((need_w + wth - 1) / wth);
   if (n_tie > n_theta) n_tie = n_theta;
-  // t* = index of the n_tie-th key equal to theta (ascending t); warp segments
-  const int seg = ((n + NW * 32 - 1) / (NW * 32)) * 32;
-  const int lo = w * seg, hi = min(n, lo + seg);
-  unsigned cnt = 0;
-  for (int base = lo; base < hi; base += 32) {
-    const int i = base + lane;
-    cnt += __popc(__ballot_sync(0xffffffffu, i < hi && get(i) == theta));
-  }
-  const unsigned before = warp_excl_prefix(S, cnt);
-  if (before < n_tie && before + cnt >= n_tie) {
-    unsigned seen = before;
+  if (tid == 0) S.aux = n;  // every key equal to theta is in
+  if (n_tie < n_theta) {
+    // t* = index of the n_tie-th key equal to theta (ascending t); warp segments
+    const int seg = ((n + NW * 32 - 1) / (NW * 32)) * 32;
+    const int lo = w * seg, hi = min(n, lo + seg);
+    unsigned cnt = 0;
     for (int base = lo; base < hi; base += 32) {
       const int i = base + lane;
-      const unsigned bal = __ballot_sync(0xffffffffu, i < hi && get(i) == theta);
-      if (seen + __popc(bal) >= n_tie) {
-        const unsigned want = n_tie - seen;   // 1-based rank inside this word
-        unsigned bb = bal;
-        for (unsigned k = 1; k < want; ++k) bb &= bb - 1;
-        if (lane == 0) S.aux = base + __ffs(bb) - 1;
-        break;
+      cnt += __popc(__ballot_sync(0xffffffffu, i < hi && get(i) == theta));
+    }
+    const unsigned before = warp_excl_prefix(S, cnt);
+    if (before < n_tie && before + cnt >= n_tie) {
+      unsigned seen = before;
+      for (int base = lo; base < hi; base += 32) {
+        const int i = base + lane;
+        const unsigned bal = __ballot_sync(0xffffffffu, i < hi && get(i) == theta);
+        if (seen + __popc(bal) >= n_tie) {
+          const unsigned want = n_tie - seen;   // 1-based rank inside this word
+          unsigned bb = bal;
+          for (unsigned k = 1; k < want; ++k) bb &= bb - 1;
+          if (lane == 0) S.aux = base + __ffs(bb) - 1;
+          break;
+        }
+        seen += __popc(bal);
       }
-      seen += __popc(bal);
     }
   }
   __syncthreads();
@@ -244,9 +295,11 @@ __global__ void __launch_bounds__(NT) cover_kernel(Problem P, Buffers bf) {
 }
 
 // from_scores: S comes from bf.scores as given; otherwise it is built here.
-__global__ void __launch_bounds__(NT) topk_kernel(Problem P, Buffers bf, int32_t* out_idx,
+__global__ void __launch_bounds__(NT, 1) topk_kernel(Problem P, Buffers bf, int32_t* out_idx,
                                                   int from_scores) {
-  extern __shared__ uint32_t keys_sm[];
+  extern __shared__ uint32_t dyn[];
+  uint32_t* hist = dyn;
+  uint32_t* keys_sm = dyn + HIST_WORDS;
   __shared__ SelShared S;
   const int h = blockIdx.x, b = blockIdx.y, l = blockIdx.z;
   const ReqInfo R = P.req[b];
@@ -256,24 +309,39 @@ __global__ void __launch_bounds__(NT) topk_kernel(Problem P, Buffers bf, int32_t
   const bool staged = n <= kMaxStaged;
   if (!from_scores) {
     const float* an = bf.anchor + hrow;
-    for (int i = tid; i < n; i += NT) {
+    const uint32_t* bw = bf.bits + ((size_t)l * P.Hkv + h) * P.G * P.total_words + R.word_off;
+    // each warp takes 32 consecutive keys at a time
+    for (int base = w * 32; base < n; base += NT) {
+      const int i = base + lane;
       float s;
       if (P.mode == MMSHIFT_SCORE_VOTE) {
+        // lane g holds the coverage word of group g for these 32 keys; the
+        // vote of key base+j is the number of lanes whose bit j is set
         unsigned vote = 0;
-        const uint32_t* bw = bf.bits + ((size_t)l * P.Hkv + h) * P.G * P.total_words + R.word_off + (i >> 5);
-        for (int g = 0; g < P.G; ++g) vote += (bw[(size_t)g * P.total_words] >> (i & 31)) & 1u;
-        s = __fadd_rn((float)vote, __fmul_rn(P.lambda, an[i]));  // no contraction
+        for (int g0 = 0; g0 < P.G; g0 += 32) {
+          const int g = g0 + lane;
+          const uint32_t word = g < P.G ? bw[(size_t)g * P.total_words + (base >> 5)] : 0u;
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const unsigned c = __popc(__ballot_sync(0xffffffffu, (word >> j) & 1u));
+            if (lane == j) vote += c;
+          }
+        }
+        s = i < n ? __fadd_rn((float)vote, __fmul_rn(P.lambda, an[i])) : 0.f;  // no contraction
       } else {
         float ms = 0.f;
-        for (int g = 0; g < P.G; ++g)
-          ms += bf.gmass[(((size_t)l * P.Hkv + h) * P.G + g) * P.total_T + R.tok_off + i];
+        if (i < n)
+          for (int g = 0; g < P.G; ++g)
+            ms += bf.gmass[(((size_t)l * P.Hkv + h) * P.G + g) * P.total_T + R.tok_off + i];
         s = ms;
       }
-      sc[i] = s;
-      if (staged) keys_sm[i] = ordered_key(s);
+      if (i < n) {
+        sc[i] = s;
+        if (staged) keys_sm[i] = nonneg_key(s);
+      }
     }
   } else if (staged) {
-    for (int i = tid; i < n; i += NT) keys_sm[i] = ordered_key(sc[i]);
+    for (int i = tid; i < n; i += NT) keys_sm[i] = nonneg_key(sc[i]);
   }
   __syncthreads();
   int32_t* out = out_idx + ((size_t)l * P.R + R.out_off) * P.Hkv + h;
@@ -288,7 +356,7 @@ __global__ void __launch_bounds__(NT) topk_kernel(Problem P, Buffers bf, int32_t
   }
   KeySrc get{staged ? keys_sm : nullptr, sc};
   const int nc = n - 1;  // candidates t < T-1
-  radix_select<false>(get, nc, 0ull, (unsigned)(keep - 1), 0, S);
+  radix_select<false>(get, nc, 0ull, (unsigned)(keep - 1), 0, 0.f, S, hist);
   const uint32_t theta = S.prefix;
   const unsigned n_tie = (unsigned)(keep - 1) - S.cum_n;
   // ordered compaction over warp segments
@@ -372,9 +440,9 @@ cudaError_t launch_cover(const Problem& P, const Buffers& bf, cudaStream_t st) {
   if (P.G == 0) return cudaSuccess;
   int maxT = 0;
   for (int b = 0; b < P.B; ++b) maxT = max(maxT, P.req[b].t_len);
-  const size_t smem = (size_t)min(maxT, kMaxStaged) * sizeof(uint32_t);
+  const size_t smem = (size_t)(HIST_WORDS + min(maxT, kMaxStaged)) * sizeof(uint32_t);
   cudaError_t e = cudaFuncSetAttribute(cover_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)(kMaxStaged * sizeof(uint32_t)));
+                                       (int)((HIST_WORDS + kMaxStaged) * sizeof(uint32_t)));
   if (e != cudaSuccess) return e;
   dim3 grid(P.Hkv * P.G, P.B, P.L);
   cover_kernel<<<grid, NT, smem, st>>>(P, bf);
@@ -385,9 +453,9 @@ cudaError_t launch_topk(const Problem& P, const Buffers& bf, cudaStream_t st, in
                         bool from_scores) {
   int maxT = 0;
   for (int b = 0; b < P.B; ++b) maxT = max(maxT, P.req[b].t_len);
-  const size_t smem = (size_t)min(maxT, kMaxStaged) * sizeof(uint32_t);
+  const size_t smem = (size_t)(HIST_WORDS + min(maxT, kMaxStaged)) * sizeof(uint32_t);
   cudaError_t e = cudaFuncSetAttribute(topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)(kMaxStaged * sizeof(uint32_t)));
+                                       (int)((HIST_WORDS + kMaxStaged) * sizeof(uint32_t)));
   if (e != cudaSuccess) return e;
   dim3 grid(P.Hkv, P.B, P.L);
   topk_kernel<<<grid, NT, smem, st>>>(P, bf, out_idx, from_scores ? 1 : 0);

@@ -10,9 +10,12 @@
 namespace mmshift {
 namespace umma {
 
-// Bounded spins: a wait that does not complete within this many polls gives
-// up, flags the CTA to abort and lets the kernel report a timeout.
-constexpr uint32_t kSpinLimit = 1u << 24;
+// Bounded waits: a thread polls an mbarrier at most kSpinLimit times, each
+// poll suspending it for up to kSuspendNs nanoseconds (so waiting threads do
+// not take issue slots from working ones); then it gives up, flags the CTA to
+// abort and lets the kernel report a timeout (about 4 s in the worst case).
+constexpr uint32_t kSpinLimit = 1u << 15;
+constexpr uint32_t kSuspendNs = 100000;
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -41,10 +44,10 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(kSuspendNs)
       : "memory");
   return ok != 0;
 }
@@ -54,7 +57,7 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
   for (uint32_t i = 0; i < kSpinLimit; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 255u) == 255u && *abort) return false;
+    if (*abort) return false;
   }
   *abort = 1;
   return false;

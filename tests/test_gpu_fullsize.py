@@ -1,0 +1,134 @@
+"""GPU parity at the workloads' full sizes, in the launch configuration the
+benchmark uses (every layer of the stack in one mmshift_select call), checked
+on sampled (layer, KV head) units that the oracle computes one by one.
+
+Proxies are given (seeded, from the shared generator) where masses and the
+selection are compared strictly; the sampled-proxy path the benchmark runs is
+checked on its proxies (one ulp) and on index overlap.
+"""
+import multiprocessing as mp
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2607_22586_gb300 import synth as S
+from oracle import mmshift_oracle as O
+from tests import parity as PT
+
+pytestmark = pytest.mark.gpu
+
+
+def _gen(args):
+    wl, layer = args
+    return S.make_layer(wl, layer)
+
+
+def _layers(wl, ids):
+    if len(ids) > 2:
+        with mp.get_context("spawn").Pool(min(8, len(ids))) as pool:
+            return pool.map(_gen, [(wl, l) for l in ids])
+    return [S.make_layer(wl, l) for l in ids]
+
+
+def _unit_ref(wl, li, h, layer_id, b, kvh, proxies=None):
+    """Oracle for one (request, KV head) of one layer."""
+    r = wl.n_q_heads // wl.n_kv_heads
+    cu = wl.cu_seqlens()
+    lo, hi = int(cu[b]), int(cu[b + 1])
+    kw = PT.oracle_kw(h, wl.dtype)
+    kw["layer_id"] = layer_id
+    pr = None if proxies is None else proxies[b, kvh * r:(kvh + 1) * r]
+    if proxies is None:
+        # the sampled proxies of query heads kvh*r.. are drawn with their own head ids
+        z = O.proxy_normals(h["seed"], layer_id, b, wl.n_q_heads, h["n_proxies"], wl.head_dim)
+        full = O.build_proxies(li.Qwin[b], z, h["gamma"], hi - lo, wl.dtype)
+        pr = full[kvh * r:(kvh + 1) * r]
+    return O.select_request(li.K[lo:hi, kvh:kvh + 1], li.V[lo:hi, kvh:kvh + 1],
+                            li.Qwin[b][:, kvh * r:(kvh + 1) * r], int(wl.budgets[b]), b=b,
+                            proxies=pr, **kw), lo, hi
+
+
+def _slice_head(gpu, kvh):
+    """View of the GPU outputs restricted to one KV head (keeps the layer axis)."""
+    return dict(gpu, group_mass=gpu["group_mass"][:, kvh:kvh + 1], anchor=gpu["anchor"][:, kvh:kvh + 1],
+                mass=gpu["mass"][:, kvh:kvh + 1], scores=gpu["scores"][:, kvh:kvh + 1],
+                idx=gpu["idx"][:, :, kvh:kvh + 1], out_k=gpu["out_k"][:, :, kvh:kvh + 1],
+                out_v=gpu["out_v"][:, :, kvh:kvh + 1], K=gpu["K"][:, :, kvh:kvh + 1],
+                V=gpu["V"][:, :, kvh:kvh + 1])
+
+
+def _check_units(wl, gpu, lis, layer_ids, h, units, proxies=None):
+    outs = np.concatenate([[0], np.cumsum(np.minimum(wl.budgets, wl.seq_lens))])
+    for li_pos, b, kvh in units:
+        ref, lo, hi = _unit_ref(wl, lis[li_pos], h, layer_ids[li_pos], b, kvh,
+                                None if proxies is None else proxies[li_pos])
+        g = _slice_head(gpu, kvh)
+        what = f"{wl.name} layer {layer_ids[li_pos]} req {b} head {kvh}"
+        PT.check_request(g, ref, h, lo, hi, li_pos, what, out_lo=int(outs[b]))
+        keep = min(wl.budgets[b], hi - lo)
+        PT.check_gather(g, wl, li_pos, lo, int(outs[b]), keep, hi - lo, 1)
+
+
+def test_long_context_stack_full_size():
+    """28 layers x 32768 tokens (4 images + text), all layers in one call;
+    oracle on layers 0, 14, 27 x all KV heads."""
+    wl = S.WORKLOADS["qwen7b-28l-32k"]
+    ids = list(range(wl.n_layers))
+    lis = _layers(wl, ids)
+    h = PT.hyper()
+    prox = np.stack([S.make_proxies(wl, h["n_proxies"], l) for l in ids])
+    gpu = PT.gpu_select(wl, lis, h, proxies=prox)
+    assert gpu["score_path"] == 1
+    units = [(l, 0, kvh) for l in (0, 14, 27) for kvh in range(wl.n_kv_heads)]
+    _check_units(wl, gpu, lis, ids, h, units, proxies=prox)
+
+
+def test_long_context_stack_sampled_proxies():
+    """The benchmark's own path (proxies sampled on the GPU): proxies within one
+    bf16 ulp of the oracle's and the kept sets overlapping on sampled units."""
+    wl = S.WORKLOADS["qwen7b-28l-32k"]
+    ids = [0, 13, 27]
+    lis = _layers(wl, ids)
+    h = PT.hyper(seed=7)
+    # three layers of the stack in one call keep the per-layer random streams
+    # of layers 0, 13 and 27 only if called one by one
+    for pos, l in enumerate(ids):
+        gpu = PT.gpu_select(wl, [lis[pos]], dict(h, layer_id=l))
+        for kvh in range(wl.n_kv_heads):
+            ref, lo, hi = _unit_ref(wl, lis[pos], h, l, 0, kvh)
+            r = wl.n_q_heads // wl.n_kv_heads
+            got = gpu["proxies"][0, 0, kvh * r:(kvh + 1) * r].astype(np.float64)
+            _, e = np.frexp(np.maximum(np.abs(ref["proxies"]), np.abs(got)))
+            diff = np.abs(got - ref["proxies"])
+            assert np.mean(diff > 0) <= 1e-3
+            a = set(gpu["idx"][0][:, kvh].tolist())
+            b = set(ref["idx"][:, 0].tolist())
+            assert len(a & b) >= 0.98 * len(b), f"layer {l} head {kvh}: {len(a & b)}/{len(b)}"
+
+
+def test_ragged_72b_batch_full_lengths():
+    """Hq64/Hkv8, 8 requests of 2048..24576 tokens, every request at its full
+    length; three layers in one call; oracle on a sample of (request, head)."""
+    wl = S.WORKLOADS["72b-80l-ragged"]
+    ids = [0, 40, 79]
+    lis = _layers(wl, ids)
+    h = PT.hyper(layer_id=0)
+    prox = np.stack([S.make_proxies(wl, h["n_proxies"], l) for l in ids])
+    gpu = PT.gpu_select(wl, lis, h, proxies=prox)
+    assert gpu["score_path"] == 1
+    units = [(0, 0, 0), (0, 7, 5), (1, 3, 2), (1, 5, 7), (2, 6, 1), (2, 1, 4)]
+    _check_units(wl, gpu, lis, ids, h, units, proxies=prox)
+
+
+@pytest.mark.parametrize("window", S.SWEEP_8K_WINDOWS)
+@pytest.mark.parametrize("budget", S.SWEEP_8K_BUDGETS)
+def test_stack_8k_window_budget_sweep(window, budget):
+    wl = S.WORKLOADS["qwen7b-28l-8k"].replace(window=window, budgets=(budget,))
+    ids = [0, 27]
+    lis = _layers(wl, ids)
+    h = PT.hyper()
+    prox = np.stack([S.make_proxies(wl, h["n_proxies"], l) for l in ids])
+    gpu = PT.gpu_select(wl, lis, h, proxies=prox)
+    units = [(0, 0, (window // 16) % wl.n_kv_heads), (1, 0, budget % wl.n_kv_heads)]
+    _check_units(wl, gpu, lis, ids, h, units, proxies=prox)
