@@ -25,11 +25,14 @@
 namespace mmshift {
 namespace {
 
-constexpr int NT = 512;           // threads per selection CTA
+constexpr int NT = 512;           // threads per top-k CTA
 constexpr int NW = NT / 32;
+constexpr int NTC = 256;          // threads per coverage CTA
 constexpr int NBIN = 256;
-constexpr int kMaxStaged = 40960; // keys staged in shared memory (160 KB)
-constexpr int HIST_WORDS = 3 * NW * NBIN;  // per-warp count / weight-lo / weight-hi
+constexpr int kMaxStaged = 40960; // top-k keys staged in shared memory (160 KB)
+
+template <int NTH>
+constexpr int hist_words() { return 3 * (NTH / 32) * NBIN; }  // per-warp count / weight lo / hi
 
 __device__ __forceinline__ uint32_t ordered_key(float x) {
   uint32_t u = __float_as_uint(x + 0.0f);  // -0 -> +0
@@ -43,17 +46,20 @@ __device__ __forceinline__ uint32_t nonneg_key(float x) {
   return ordered_key(fmaxf(x, 0.f));
 }
 
+template <int NTH>
 struct SelShared {
   unsigned long long total;
-  unsigned long long wsum[NW];
-  unsigned int wcnt[NW];
+  unsigned long long wsum[NTH / 32];
+  unsigned int wcnt[NTH / 32];
+  unsigned long long bin_w[NBIN];
+  unsigned int bin_n[NBIN];
   unsigned long long cum_w;
   unsigned int cum_n;
   unsigned int digit;
   unsigned int prefix;
   unsigned int n_theta;
+  unsigned int max_key;
   int aux;
-  float fsum;
 };
 
 // Key source: shared memory when staged, else recomputed from global floats.
@@ -61,7 +67,7 @@ struct KeySrc {
   const uint32_t* smem;
   const float* gmem;
   __device__ __forceinline__ uint32_t operator()(int i) const {
-    return smem ? smem[i] : nonneg_key(gmem[i]);
+    return smem ? smem[i] : nonneg_key(__ldg(gmem + i));
   }
 };
 
@@ -71,7 +77,8 @@ __device__ __forceinline__ unsigned long long fx_weight(uint32_t key, int shift)
 }
 
 // Block-wide exclusive scan of one unsigned per warp (warp totals in S.wcnt).
-__device__ __forceinline__ unsigned warp_excl_prefix(SelShared& S, unsigned mine) {
+template <int NTH>
+__device__ __forceinline__ unsigned warp_excl_prefix(SelShared<NTH>& S, unsigned mine) {
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (lane == 0) S.wcnt[w] = mine;
   __syncthreads();
@@ -81,48 +88,45 @@ __device__ __forceinline__ unsigned warp_excl_prefix(SelShared& S, unsigned mine
   return before;
 }
 
-// Smallest prefix of the (key desc, index asc) order whose cumulative weight
-// is >= target_w and whose length is >= target_n (all keys >= 0x80000000,
-// i.e. of non-negative values). On return S.prefix is the key theta of the
-// prefix's last element, S.cum_w / S.cum_n the weight / count of keys above
-// theta and S.n_theta the number of keys equal to theta. `hist` is
-// HIST_WORDS words of shared memory.
-//
-// Weighted mode: target_w is derived from the exact fixed-point total, summed in
-// the first pass: target_w = min(total, ceil(tau * total)); S.total holds it.
-template <bool WEIGHTED>
-__device__ void radix_select(const KeySrc& get, int n, unsigned long long target_w,
-                             unsigned target_n, int shift, float tau, SelShared& S,
-                             uint32_t* hist) {
+// One digit pass: per-warp histograms of the keys matching `prefix` above
+// bit `hs`, digit = bits [sh, hs). Weighted: also the weights, and in the
+// first pass the exact total (returned through S.wsum) and the largest key.
+template <bool WEIGHTED, int NTH>
+__device__ __forceinline__ void digit_histogram(const KeySrc& get, int n, uint32_t prefix, int sh,
+                                                int hs, uint32_t dmask, int shift, bool first,
+                                                SelShared<NTH>& S, uint32_t* hist) {
+  constexpr int NWH = NTH / 32;
   const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
   uint32_t* hn = hist + w * NBIN;
-  uint32_t* hlo = hist + (NW + w) * NBIN;
-  uint32_t* hhi = hist + (2 * NW + w) * NBIN;
-  if (tid == 0) { S.cum_w = 0; S.cum_n = 0; }
-  uint32_t prefix = 0x80000000u;
-  constexpr int kSh[4] = {23, 15, 7, 0};
-  constexpr int kWid[4] = {8, 8, 8, 7};
-#pragma unroll 1
-  for (int pass = 0; pass < 4; ++pass) {
-    const int sh = kSh[pass], hs = sh + kWid[pass];
-    const uint32_t dmask = (1u << kWid[pass]) - 1u;
-    for (int i = lane; i < NBIN; i += 32) {
-      hn[i] = 0;
-      if (WEIGHTED) { hlo[i] = 0; hhi[i] = 0; }
+  uint32_t* hlo = hist + (NWH + w) * NBIN;
+  uint32_t* hhi = hist + (2 * NWH + w) * NBIN;
+  for (int i = lane; i < NBIN; i += 32) {
+    hn[i] = 0;
+    if (WEIGHTED) { hlo[i] = 0; hhi[i] = 0; }
+  }
+  __syncwarp();
+  unsigned long long tot = 0;
+  uint32_t kmax = 0;
+  constexpr int U = 8;  // independent loads in flight per thread
+  for (int base = 0; base < n; base += U * NTH) {
+    uint32_t kk[U];
+#pragma unroll
+    for (int j = 0; j < U; ++j) {
+      const int i = base + j * NTH + tid;
+      kk[j] = i < n ? get(i) : 0u;
     }
-    __syncwarp();
-    unsigned long long tot = 0;
-    for (int base = 0; base < n; base += NT) {
-      const int i = base + tid;
-      const uint32_t k = i < n ? get(i) : 0u;
+#pragma unroll
+    for (int j = 0; j < U; ++j) {
+      const int i = base + j * NTH + tid;
+      const uint32_t k = kk[j];
       const bool take = i < n && (k >> hs) == (prefix >> hs);
-      if (pass > 0 && !__any_sync(0xffffffffu, take)) continue;
+      if (!first && !__any_sync(0xffffffffu, take)) continue;
       if (take) {
         const uint32_t d = (k >> sh) & dmask;
         atomicAdd(&hn[d], 1u);
         if (WEIGHTED) {
           const unsigned long long wt = fx_weight(k, shift);
-          if (pass == 0) tot += wt;
+          if (first) { tot += wt; kmax = max(kmax, k); }
           const uint32_t lo = (uint32_t)wt;
           uint32_t hi = (uint32_t)(wt >> 32);
           if (lo) {
@@ -133,77 +137,119 @@ __device__ void radix_select(const KeySrc& get, int n, unsigned long long target
         }
       }
     }
-    if (WEIGHTED && pass == 0) {
-      for (int off = 16; off; off >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, off);
-      if (lane == 0) S.wsum[w] = tot;
+  }
+  if (WEIGHTED && first) {
+    for (int off = 16; off; off >>= 1) {
+      tot += __shfl_xor_sync(0xffffffffu, tot, off);
+      kmax = max(kmax, __shfl_xor_sync(0xffffffffu, kmax, off));
     }
-    __syncthreads();
+    if (lane == 0) { S.wsum[w] = tot; S.wcnt[w] = kmax; }
+  }
+  __syncthreads();
+  // combine the per-warp histograms: bin totals in shared memory
+  for (int d = tid; d < NBIN; d += NTH) {
+    unsigned long long wsum = 0;
+    unsigned nsum = 0;
+    for (int ww = 0; ww < NWH; ++ww) {
+      nsum += hist[ww * NBIN + d];
+      if (WEIGHTED)
+        wsum += (unsigned long long)hist[(NWH + ww) * NBIN + d] +
+                ((unsigned long long)hist[(2 * NWH + ww) * NBIN + d] << 32);
+    }
+    S.bin_n[d] = nsum;
+    S.bin_w[d] = wsum;
+  }
+  __syncthreads();
+}
+
+// Pick the digit where the (key desc) cumulative weight / count first reaches
+// the targets; warp 0 only. Lane L owns digits 255-8L .. 248-8L.
+template <bool WEIGHTED, int NTH>
+__device__ __forceinline__ void digit_scan(unsigned long long target_w, unsigned target_n,
+                                           SelShared<NTH>& S) {
+  const int lane = threadIdx.x & 31;
+  unsigned long long sw = 0;
+  unsigned sn = 0;
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const int d = 255 - 8 * lane - k;
+    sw += S.bin_w[d];
+    sn += S.bin_n[d];
+  }
+  unsigned long long iw = sw;
+  unsigned in = sn;
+  for (int off = 1; off < 32; off <<= 1) {
+    const unsigned long long tw = __shfl_up_sync(0xffffffffu, iw, off);
+    const unsigned tn = __shfl_up_sync(0xffffffffu, in, off);
+    if (lane >= off) { iw += tw; in += tn; }
+  }
+  const unsigned long long cw = S.cum_w;
+  const unsigned cn = S.cum_n;
+  const bool hit = (!WEIGHTED || cw + iw >= target_w) && cn + in >= target_n;
+  const unsigned ball = __ballot_sync(0xffffffffu, hit);
+  const int f = ball ? __ffs(ball) - 1 : 31;
+  if (lane == f) {
+    unsigned long long c_w = cw + iw - sw;
+    unsigned c_n = cn + in - sn;
+    int chosen = 255 - 8 * lane - 7;
+    for (int k = 0; k < 8; ++k) {
+      const int d = 255 - 8 * lane - k;
+      if ((!WEIGHTED || c_w + S.bin_w[d] >= target_w) && c_n + S.bin_n[d] >= target_n) {
+        chosen = d;
+        break;
+      }
+      if (k < 7) { c_w += S.bin_w[d]; c_n += S.bin_n[d]; }
+    }
+    S.cum_w = c_w;
+    S.cum_n = c_n;
+    S.digit = (unsigned)chosen;
+    S.n_theta = S.bin_n[chosen];
+  }
+}
+
+// Smallest prefix of the (key desc, index asc) order whose cumulative weight
+// is >= target_w and whose length is >= target_n (all keys are of
+// non-negative values). On return S.prefix is the key theta of the prefix's
+// last element, S.cum_w / S.cum_n the weight / count of keys above theta and
+// S.n_theta the number of keys equal to theta. Weighted mode: target_w is
+// min(total, ceil(tau * total)) of the exact fixed-point total (S.total), and
+// *shift is lowered (and the first pass redone) if 2^shift units could
+// overflow 64 bits. `hist` is hist_words<NTH>() words of shared memory.
+template <bool WEIGHTED, int NTH>
+__device__ void radix_select(const KeySrc& get, int n, unsigned long long target_w,
+                             unsigned target_n, int* shift, float tau, SelShared<NTH>& S,
+                             uint32_t* hist) {
+  constexpr int NWH = NTH / 32;
+  const int tid = threadIdx.x;
+  if (tid == 0) { S.cum_w = 0; S.cum_n = 0; }
+  uint32_t prefix = 0x80000000u;
+  constexpr int kSh[4] = {23, 15, 7, 0};
+  constexpr int kWid[4] = {8, 8, 8, 7};
+#pragma unroll 1
+  for (int pass = 0; pass < 4; ++pass) {
+    const int sh = kSh[pass], hs = sh + kWid[pass];
+    const uint32_t dmask = (1u << kWid[pass]) - 1u;
+    digit_histogram<WEIGHTED, NTH>(get, n, prefix, sh, hs, dmask, WEIGHTED ? *shift : 0,
+                                   pass == 0, S, hist);
     if (WEIGHTED && pass == 0) {
+      uint32_t kmax = 0;
+      for (int i = 0; i < NWH; ++i) kmax = max(kmax, S.wcnt[i]);
+      int e = 0;
+      frexpf(key_value(kmax), &e);              // values < 2^e
+      int lg = 0;
+      while ((1 << lg) < n) ++lg;               // n <= 2^lg
+      if (e + lg + *shift > 63) {               // n * max * 2^shift could overflow
+        *shift = max(0, 63 - e - lg);
+        __syncthreads();
+        digit_histogram<WEIGHTED, NTH>(get, n, prefix, sh, hs, dmask, *shift, true, S, hist);
+      }
       unsigned long long total = 0;
-      for (int i = 0; i < NW; ++i) total += S.wsum[i];
-      unsigned long long t = (unsigned long long)ceil((double)tau * (double)total);
+      for (int i = 0; i < NWH; ++i) total += S.wsum[i];
+      const unsigned long long t = (unsigned long long)ceil((double)tau * (double)total);
       target_w = t > total ? total : t;
       if (tid == 0) S.total = total;
     }
-    if (tid < 32) {
-      // lane L owns digits 255-8L .. 248-8L, scanned from the top
-      unsigned long long bw[8];
-      unsigned bn[8];
-      unsigned long long sw = 0;
-      unsigned sn = 0;
-#pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        const int d = 255 - 8 * lane - k;
-        unsigned long long wsum = 0;
-        unsigned nsum = 0;
-        for (int ww = 0; ww < NW; ++ww) {
-          nsum += hist[ww * NBIN + d];
-          if (WEIGHTED)
-            wsum += (unsigned long long)hist[(NW + ww) * NBIN + d] +
-                    ((unsigned long long)hist[(2 * NW + ww) * NBIN + d] << 32);
-        }
-        bw[k] = wsum;
-        bn[k] = nsum;
-        sw += wsum;
-        sn += nsum;
-      }
-      unsigned long long iw = sw;
-      unsigned in = sn;
-      for (int off = 1; off < 32; off <<= 1) {
-        const unsigned long long tw = __shfl_up_sync(0xffffffffu, iw, off);
-        const unsigned tn = __shfl_up_sync(0xffffffffu, in, off);
-        if (lane >= off) { iw += tw; in += tn; }
-      }
-      const unsigned long long cw = S.cum_w;
-      const unsigned cn = S.cum_n;
-      const bool hit = (!WEIGHTED || cw + iw >= target_w) && cn + in >= target_n;
-      const unsigned ball = __ballot_sync(0xffffffffu, hit);
-      const int f = ball ? __ffs(ball) - 1 : 31;
-      if (lane == f) {
-        unsigned long long c_w = cw + iw - sw;
-        unsigned c_n = cn + in - sn;
-        int chosen = 7;
-        unsigned n_ch = bn[7];
-        bool found = false;
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-          if (!found) {
-            if ((!WEIGHTED || c_w + bw[k] >= target_w) && c_n + bn[k] >= target_n) {
-              chosen = k;
-              n_ch = bn[k];
-              found = true;
-            } else if (k < 7) {
-              c_w += bw[k];
-              c_n += bn[k];
-            }
-          }
-        }
-        S.cum_w = c_w;
-        S.cum_n = c_n;
-        S.digit = (unsigned)(255 - 8 * lane - chosen);
-        S.n_theta = n_ch;
-      }
-    }
+    if (tid < 32) digit_scan<WEIGHTED, NTH>(target_w, target_n, S);
     __syncthreads();
     prefix |= (S.digit & dmask) << sh;
     __syncthreads();
@@ -212,57 +258,42 @@ __device__ void radix_select(const KeySrc& get, int n, unsigned long long target
   __syncthreads();
 }
 
-__global__ void __launch_bounds__(NT, 1) cover_kernel(Problem P, Buffers bf) {
+__global__ void __launch_bounds__(NTC, 4) cover_kernel(Problem P, Buffers bf) {
   extern __shared__ uint32_t dyn[];
   uint32_t* hist = dyn;
-  uint32_t* keys_sm = dyn + HIST_WORDS;
-  __shared__ SelShared S;
+  __shared__ SelShared<NTC> S;
+  constexpr int NWC = NTC / 32;
   const int g = blockIdx.x % P.G, h = blockIdx.x / P.G, b = blockIdx.y, l = blockIdx.z;
   const ReqInfo R = P.req[b];
   const int n = R.t_len, tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
   const size_t row = ((size_t)l * P.Hkv + h) * P.G + g;
   const float* m = bf.gmass + row * P.total_T + R.tok_off;
-  const bool staged = n <= kMaxStaged;
-  // stage keys and sum the masses (float, only to choose the fixed point)
-  float fs = 0.f;
-  for (int i = tid; i < n; i += NT) {
-    const float x = fmaxf(m[i], 0.f);
-    if (staged) keys_sm[i] = ordered_key(x);
-    fs += x;
-  }
-  for (int off = 16; off; off >>= 1) fs += __shfl_xor_sync(0xffffffffu, fs, off);
-  if (lane == 0) S.wsum[w] = __float_as_uint(fs);
-  __syncthreads();
-  if (tid == 0) {
-    float t = 0.f;
-    for (int i = 0; i < NW; ++i) t += __uint_as_float((unsigned)S.wsum[i]);
-    S.fsum = t;
-  }
-  __syncthreads();
-  int e = 0;
-  frexpf(S.fsum + 1.0f, &e);               // S.fsum + 1 < 2^e
-  const int shift = max(0, min(40, 60 - e));
-  KeySrc get{staged ? keys_sm : nullptr, m};
-  radix_select<true>(get, n, 0ull, 1u, shift, P.tau, S, hist);
+  // masses are read from L2 in every pass (the working set of the resident
+  // CTAs fits), which keeps shared memory small and four CTAs per SM
+  KeySrc get{nullptr, m};
+  int shift = 40;
+  radix_select<true, NTC>(get, n, 0ull, 1u, &shift, P.tau, S, hist);
   const uint32_t theta = S.prefix;
   const unsigned n_theta = S.n_theta;
-  const unsigned long long target = min(S.total, (unsigned long long)ceil((double)P.tau * (double)S.total));
+  const unsigned long long target =
+      min(S.total, (unsigned long long)ceil((double)P.tau * (double)S.total));
   const unsigned long long wth = fx_weight(theta, shift);
   const unsigned long long need_w = target > S.cum_w ? target - S.cum_w : 0ull;
   unsigned n_tie = 1;
   if (need_w > 0 && wth > 0) n_tie = (unsigned)((need_w + wth - 1) / wth);
   if (n_tie > n_theta) n_tie = n_theta;
   if (tid == 0) S.aux = n;  // every key equal to theta is in
+  __syncthreads();
   if (n_tie < n_theta) {
     // t* = index of the n_tie-th key equal to theta (ascending t); warp segments
-    const int seg = ((n + NW * 32 - 1) / (NW * 32)) * 32;
+    const int seg = ((n + NWC * 32 - 1) / (NWC * 32)) * 32;
     const int lo = w * seg, hi = min(n, lo + seg);
     unsigned cnt = 0;
     for (int base = lo; base < hi; base += 32) {
       const int i = base + lane;
       cnt += __popc(__ballot_sync(0xffffffffu, i < hi && get(i) == theta));
     }
-    const unsigned before = warp_excl_prefix(S, cnt);
+    const unsigned before = warp_excl_prefix<NTC>(S, cnt);
     if (before < n_tie && before + cnt >= n_tie) {
       unsigned seen = before;
       for (int base = lo; base < hi; base += 32) {
@@ -282,25 +313,31 @@ __global__ void __launch_bounds__(NT, 1) cover_kernel(Problem P, Buffers bf) {
   __syncthreads();
   const int tstar = S.aux;
   uint32_t* bits = bf.bits + row * P.total_words + R.word_off;
-  for (int base = w * 32; base < n; base += NT) {
-    const int i = base + lane;
-    bool mem = false;
-    if (i < n) {
-      const uint32_t k = get(i);
-      mem = k > theta || (k == theta && i <= tstar);
+  constexpr int U = 8;
+  for (int base = w * 32; base < n; base += U * NTC) {
+    uint32_t kk[U];
+#pragma unroll
+    for (int j = 0; j < U; ++j) {
+      const int i = base + j * NTC + lane;
+      kk[j] = i < n ? get(i) : 0u;
     }
-    const unsigned word = __ballot_sync(0xffffffffu, mem);
-    if (lane == 0) bits[base >> 5] = word;
+#pragma unroll
+    for (int j = 0; j < U; ++j) {
+      const int i = base + j * NTC + lane;
+      const bool mem = i < n && (kk[j] > theta || (kk[j] == theta && i <= tstar));
+      const unsigned word = __ballot_sync(0xffffffffu, mem);
+      if (lane == 0 && base + j * NTC < n) bits[(base + j * NTC) >> 5] = word;
+    }
   }
 }
 
 // from_scores: S comes from bf.scores as given; otherwise it is built here.
 __global__ void __launch_bounds__(NT, 1) topk_kernel(Problem P, Buffers bf, int32_t* out_idx,
-                                                  int from_scores) {
+                                                     int from_scores) {
   extern __shared__ uint32_t dyn[];
   uint32_t* hist = dyn;
-  uint32_t* keys_sm = dyn + HIST_WORDS;
-  __shared__ SelShared S;
+  uint32_t* keys_sm = dyn + hist_words<NT>();
+  __shared__ SelShared<NT> S;
   const int h = blockIdx.x, b = blockIdx.y, l = blockIdx.z;
   const ReqInfo R = P.req[b];
   const int n = R.t_len, tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
@@ -356,7 +393,7 @@ __global__ void __launch_bounds__(NT, 1) topk_kernel(Problem P, Buffers bf, int3
   }
   KeySrc get{staged ? keys_sm : nullptr, sc};
   const int nc = n - 1;  // candidates t < T-1
-  radix_select<false>(get, nc, 0ull, (unsigned)(keep - 1), 0, 0.f, S, hist);
+  radix_select<false, NT>(get, nc, 0ull, (unsigned)(keep - 1), nullptr, 0.f, S, hist);
   const uint32_t theta = S.prefix;
   const unsigned n_tie = (unsigned)(keep - 1) - S.cum_n;
   // ordered compaction over warp segments
@@ -369,8 +406,8 @@ __global__ void __launch_bounds__(NT, 1) topk_kernel(Problem P, Buffers bf, int3
     c_gt += __popc(__ballot_sync(0xffffffffu, i < hi && k > theta));
     c_tie += __popc(__ballot_sync(0xffffffffu, i < hi && k == theta));
   }
-  const unsigned gt_before = warp_excl_prefix(S, c_gt);
-  unsigned tie_before = warp_excl_prefix(S, c_tie);
+  const unsigned gt_before = warp_excl_prefix<NT>(S, c_gt);
+  unsigned tie_before = warp_excl_prefix<NT>(S, c_tie);
   unsigned pos = gt_before + min(tie_before, n_tie);
   const unsigned lt = (1u << lane) - 1u;
   for (int base = lo; base < hi; base += 32) {
@@ -438,14 +475,9 @@ cudaError_t launch_mass_sum(const Problem& P, const Buffers& bf, cudaStream_t st
 
 cudaError_t launch_cover(const Problem& P, const Buffers& bf, cudaStream_t st) {
   if (P.G == 0) return cudaSuccess;
-  int maxT = 0;
-  for (int b = 0; b < P.B; ++b) maxT = max(maxT, P.req[b].t_len);
-  const size_t smem = (size_t)(HIST_WORDS + min(maxT, kMaxStaged)) * sizeof(uint32_t);
-  cudaError_t e = cudaFuncSetAttribute(cover_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)((HIST_WORDS + kMaxStaged) * sizeof(uint32_t)));
-  if (e != cudaSuccess) return e;
+  const size_t smem = (size_t)hist_words<NTC>() * sizeof(uint32_t);
   dim3 grid(P.Hkv * P.G, P.B, P.L);
-  cover_kernel<<<grid, NT, smem, st>>>(P, bf);
+  cover_kernel<<<grid, NTC, smem, st>>>(P, bf);
   return cudaGetLastError();
 }
 
@@ -453,9 +485,9 @@ cudaError_t launch_topk(const Problem& P, const Buffers& bf, cudaStream_t st, in
                         bool from_scores) {
   int maxT = 0;
   for (int b = 0; b < P.B; ++b) maxT = max(maxT, P.req[b].t_len);
-  const size_t smem = (size_t)(HIST_WORDS + min(maxT, kMaxStaged)) * sizeof(uint32_t);
+  const size_t smem = (size_t)(hist_words<NT>() + min(maxT, kMaxStaged)) * sizeof(uint32_t);
   cudaError_t e = cudaFuncSetAttribute(topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)((HIST_WORDS + kMaxStaged) * sizeof(uint32_t)));
+                                       (int)((hist_words<NT>() + kMaxStaged) * sizeof(uint32_t)));
   if (e != cudaSuccess) return e;
   dim3 grid(P.Hkv, P.B, P.L);
   topk_kernel<<<grid, NT, smem, st>>>(P, bf, out_idx, from_scores ? 1 : 0);
