@@ -22,9 +22,9 @@
 //   K tile = N operand (M=128, N=128, two MMAs); the accumulator lane is a
 //   proxy row, so each thread keeps its row's running (max, sum of exp2) over
 //   the 128 keys of a tile without any cross-thread reduction. The running max
-//   is only raised when a 32-key chunk's sum would exceed 2^64 (or on the
-//   first chunk), so the common path is one FFMA, one MUFU.EX2 and one FADD
-//   per logit.
+//   is only raised when a 32-key chunk's sum would exceed 2^100 (or on the
+//   first chunk), and it is carried over from split to split of the same
+//   block, so the common path is one FFMA, one MUFU.EX2 and one FADD per logit.
 // Mass pass (PASS 2): K tile = M operand (128 keys), stationary = up to 256
 //   proxy rows holding whole groups as the N operand; the accumulator lane is
 //   a key, so each thread sums exp2(x - c_row) over the columns of a group in
@@ -130,7 +130,8 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
 // c0..c0+31 of the tile; columns >= nvalid are past the split and ignored).
 // m is the running max of the log2-scaled logits, z the sum of exp2(x - m).
 // The max is only raised when the chunk's sum relative to it would exceed
-// 2^64 (or on the first chunk), so the common path is FFMA + EX2 + FADD.
+// 2^100 (or on the first chunk), so the common path is FFMA + EX2 + FADD; z
+// stays below 2^127 over the 32 chunks of a key split.
 __device__ __forceinline__ void softmax_chunk(float (&v)[32], int c0, int nvalid, float alpha,
                                               float& m, float& z) {
   if (nvalid < c0 + 32) {
@@ -148,7 +149,7 @@ __device__ __forceinline__ void softmax_chunk(float (&v)[32], int c0, int nvalid
     s3 += fast_exp2(fmaf(v[j + 3], alpha, nm));
   }
   float zc = (s0 + s1) + (s2 + s3);
-  if (!(zc <= 1.8446744e19f)) {  // first chunk, overflow risk or NaN: raise the max
+  if (!(zc <= 1.2676506e30f)) {  // first chunk, sum above 2^100 or NaN: raise the max
     float cm = -INFINITY;
 #pragma unroll
     for (int j = 0; j < 32; ++j) cm = fmaxf(cm, v[j] * alpha);
@@ -368,11 +369,16 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     const int lrow = q * 32 + lane;       // accumulator lane: proxy row (1) / key (2)
     const float alpha = P.alpha;
     uint32_t ntile = 0;                   // tiles seen, in the MMA's order
+    long long prev = -1;
+    float m_run = -INFINITY;              // softmax pass: reference max of this thread's row
     for (int sr = s_begin; sr < s_end; ++sr) {
       const int u = sr * S.ntiles + my_tile;
       const Unit x = decode(P, S, u);
       const ReqInfo R = P.req[x.b];
-      float m_run = -INFINITY, z_run = 0.f;  // softmax pass state of this thread's row
+      const long long key = block_key(P, S, x);
+      if (key != prev) m_run = -INFINITY;  // a new row: no reference yet
+      prev = key;
+      float z_run = 0.f;                   // sum of exp2(x - m_run) over this split
       Block blk{};
       const float* cv = nullptr;
       if (PASS == 2) {
