@@ -41,6 +41,15 @@ if ROOT not in sys.path:
 from paper_2607_22586_gb300 import synth as S  # noqa: E402
 
 METRIC = "prompt tokens selected/sec per layer + % of GB300 HBM roofline (bytes read/time)"
+SFU_EX2_PER_SM_CLK = 32          # MUFU.EX2 lanes per SM per clock on GB300 (measured ~31)
+
+# DRAM traffic (read + write) of the two scoring kernels per launch of the
+# default workload, from one ncu capture of a 4-layer slice scaled by 7 to the
+# 28 layers (traffic grows with the layers; profiles/kernels_qwen7b-32k-4layers
+# _full-set.md). It describes the score_umma.cu it was measured on only.
+SCORE_TRAFFIC = {"source_sha256_16": "88d5d81df09ba7fb", "workload": "qwen7b-28l-32k",
+                 "proxies": "paper", "softmax_pass": 7 * (157.078784e6 + 19.625984e6),
+                 "mass_pass": 7 * (156.657408e6 + 46.612224e6)}
 UNIT = "tokens/s/layer"
 SM_COUNT = 152
 FP32_LANES_PER_SM = 128
@@ -181,6 +190,22 @@ def algorithmic(wl, hyper):
     rows = hyper["n_proxies"] * r + r       # proxies of the r query heads + anchor rows
     pass_flops = 2.0 * d * rows * T * hkv * L
     return k_read + gather, k_read, pass_flops
+
+
+def score_traffic(wl, args, kernel):
+    """DRAM bytes per launch of a scoring kernel from the recorded capture, or
+    None if the kernel source or the workload differ from the captured ones."""
+    import hashlib
+    src = os.path.join(ROOT, "paper_2607_22586_gb300", "csrc", "score_umma.cu")
+    try:
+        with open(src, "rb") as f:
+            digest = hashlib.sha256(f.read()).hexdigest()[:16]
+    except OSError:
+        return None
+    t = SCORE_TRAFFIC
+    if digest != t["source_sha256_16"] or wl.name != t["workload"] or args.proxies != t["proxies"]:
+        return None
+    return t.get(kernel)
 
 
 def run_reference(args, wl):
@@ -340,9 +365,15 @@ def run_gpu(args, wl):
     if umma:
         achieved = pass_flops / (dom_ms * 1e-3) / 1e12
         peak = float(peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]))
+        mhz = float(peaks.get("sm_max_mhz", 2070.0))
+        sfu_peak = SFU_EX2_PER_SM_CLK * SM_COUNT * mhz * 1e6
+        exps = pass_flops / (2.0 * wl.head_dim)          # one exp2 per logit
         roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                "frac": achieved / peak, "traffic": None, "kernel": dom,
-                "peak_kind": f"bf16 dense, sustained ({peak_src})"}
+                "frac": achieved / peak, "traffic": score_traffic(wl, args, dom), "kernel": dom,
+                "peak_kind": f"bf16 dense, sustained ({peak_src})",
+                "sfu": {"achieved": exps / (dom_ms * 1e-3), "peak": sfu_peak, "unit": "exp2/s",
+                        "frac": exps / (dom_ms * 1e-3) / sfu_peak,
+                        "peak_kind": f"{SFU_EX2_PER_SM_CLK} MUFU.EX2/clk/SM x {SM_COUNT} SMs x {mhz:.0f} MHz"}}
     else:
         achieved = pass_flops / (dom_ms * 1e-3) / 1e12
         mhz = float(peaks.get("sm_max_mhz", 2070.0))
