@@ -118,7 +118,8 @@ struct Smem {
   static constexpr int STAT_BYTES = CH * SROWS * 128;
   static constexpr int STAGE_BYTES = CH * BK * 128;
   static constexpr int RING_BYTES = NSTAGE * STAGE_BYTES;
-  static constexpr int DYN_BYTES = 1024 + STAT_BYTES + RING_BYTES;
+  static constexpr int CS_BYTES = (NEPI / 32) * SROWS * 4;    // per-warp normaliser copies
+  static constexpr int DYN_BYTES = 1024 + STAT_BYTES + RING_BYTES + CS_BYTES;
 };
 
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
@@ -173,11 +174,12 @@ __device__ __forceinline__ void softmax_chunk(float (&v)[32], int c0, int nvalid
   z += zc;
 }
 
-__device__ __forceinline__ void load_c16(const float* __restrict__ c, float (&cv)[16]) {
+// 16 consecutive row normalisers from the warp's shared-memory copy.
+__device__ __forceinline__ void load_c16(const float* c, float (&cv)[16]) {
   const float4* c4 = reinterpret_cast<const float4*>(c);
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    const float4 t = __ldg(c4 + i);
+    const float4 t = c4[i];
     cv[4 * i] = t.x; cv[4 * i + 1] = t.y; cv[4 * i + 2] = t.z; cv[4 * i + 3] = t.w;
   }
 }
@@ -195,11 +197,21 @@ __device__ __forceinline__ void mass_chunk(const float (&v)[16], const float (&c
 
 // Sum over the ncols (multiple of 16) accumulator columns of one group:
 // sum_j exp2(acc_j * alpha - c_j), four partial sums added in a fixed order.
-__device__ __forceinline__ float group_sum(uint32_t tcol, const float* __restrict__ c, int ncols,
-                                           float alpha) {
+// c points at the warp's shared-memory copy of the block's normalisers.
+__device__ __forceinline__ float group_sum(uint32_t tcol, const float* c, int ncols, float alpha) {
   float a[4] = {0.f, 0.f, 0.f, 0.f};
+  int cc = 0;
 #pragma unroll 1
-  for (int cc = 0; cc < ncols; cc += 16) {
+  for (; cc + 32 <= ncols; cc += 32) {
+    float v[32], cv[16];
+    tmem_ld32(tcol + cc, v);
+    load_c16(c + cc, cv);
+    tmem_wait_ld();
+    mass_chunk(*reinterpret_cast<float(*)[16]>(v), cv, alpha, a);
+    load_c16(c + cc + 16, cv);
+    mass_chunk(*reinterpret_cast<float(*)[16]>(v + 16), cv, alpha, a);
+  }
+  if (cc < ncols) {
     float v[16], cv[16];
     tmem_ld16(tcol + cc, v);
     load_c16(c + cc, cv);
@@ -220,6 +232,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
   unsigned char* stat = sm;
   unsigned char* ring = sm + SM::STAT_BYTES;
+  float* cs_all = reinterpret_cast<float*>(ring + SM::RING_BYTES);
   __shared__ uint64_t full[NSTAGE], empty[NSTAGE], sfull, sempty, tfull[2], tempty[2];
   __shared__ uint32_t tbase;
   __shared__ int abort_flag;
@@ -369,7 +382,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     const int lrow = q * 32 + lane;       // accumulator lane: proxy row (1) / key (2)
     const float alpha = P.alpha;
     uint32_t ntile = 0;                   // tiles seen, in the MMA's order
-    long long prev = -1;
+    long long prev = -1, prev_blk = -1;
     float m_run = -INFINITY;              // softmax pass: reference max of this thread's row
     for (int sr = s_begin; sr < s_end; ++sr) {
       const int u = sr * S.ntiles + my_tile;
@@ -380,10 +393,16 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       prev = key;
       float z_run = 0.f;                   // sum of exp2(x - m_run) over this split
       Block blk{};
-      const float* cv = nullptr;
+      const float* cv = cs_all + ew * SROWS;   // this warp's copy of the block's normalisers
       if (PASS == 2) {
         blk = mass_block(P, S, x.tile);
-        cv = bf.cvals + (((size_t)x.l * P.B + x.b) * P.Hkv + x.h) * P.Prows_pad + blk.row0;
+        if (key != prev_blk) {
+          const float* src = bf.cvals + (((size_t)x.l * P.B + x.b) * P.Hkv + x.h) * P.Prows_pad + blk.row0;
+          __syncwarp();
+          for (int i = lane; i < blk.rows; i += 32) cs_all[ew * SROWS + i] = src[i];
+          __syncwarp();
+          prev_blk = key;
+        }
       }
       bool ok = true;
       for (int kt = x.t0; kt < x.t1; kt += BK, ++ntile) {
