@@ -142,10 +142,12 @@ mmshift_status mmshift_workspace_size(const mmshift_shape* s, const mmshift_para
 
 /* Step 1 alone (Section 3.2.1, Appendix A.4): per (request, query head,
  * dimension) mean and unbiased std over the W window queries, then
- * proxies[b, hq, i, j] = mu + gamma * sigma * z with z ~ N(0, 1) drawn from
- * Philox4x64-10 + Box-Muller (counter (i*d/4 + j/4, hq, b, layer_id), key
- * (seed, 0)), optionally RoPE-rotated to position T_b + rope_pos_offset, and
- * rounded to dtype. proxies: [L, batch, Hq, N, d]. */
+ * proxies[b, hq, i, j] = mu + gamma * sigma * z with z ~ N(0, 1): one
+ * Philox4x64-10 draw (counter (i*d/8 + q, hq, b, layer_id), key (seed, 0))
+ * gives, as eight 32-bit uniforms ((w >> 9) + 1/2) 2^-23 and Box-Muller on
+ * consecutive pairs, dims 4q..4q+3 and d/2+4q..d/2+4q+3; then an optional
+ * RoPE rotation to position T_b + rope_pos_offset and rounding to dtype.
+ * proxies: [L, batch, Hq, N, d]. */
 mmshift_status mmshift_build_proxies(const mmshift_shape* s, const void* Qwin,
                                      const mmshift_params* p, void* proxies,
                                      mmshift_stream_t stream);

@@ -85,38 +85,45 @@ def philox4x64_10(ctr: np.ndarray, key: Sequence[int]) -> np.ndarray:
 
 
 def uniforms_from_bits(x: np.ndarray) -> np.ndarray:
-    """uint64 -> float64 uniform in (0, 1): ((x >> 11) + 1/2) * 2**-53."""
-    return ((x >> np.uint64(11)).astype(np.float64) + 0.5) * 2.0 ** -53
+    """uint32 words -> float64 uniforms in (0, 1): ((x >> 9) + 1/2) * 2**-23
+    (24 significant bits: exact in float32 too)."""
+    return ((np.asarray(x, dtype=np.uint64) >> np.uint64(9)).astype(np.float64) + 0.5) * 2.0 ** -23
 
 
 def proxy_normals(seed: int, layer_id: int, b: int, n_q_heads: int,
                   n_proxies: int, head_dim: int) -> np.ndarray:
     """Standard normals z[hq, i, j] for request b of layer ``layer_id``.
 
-    Counter of the draw covering dims 4q..4q+3 of proxy i of query head hq:
-    (i * d/4 + q, hq, b, layer_id); key (seed, 0). The four 64-bit outputs
-    give uniforms (u0, u1, u2, u3) and
-    z[4q]   = sqrt(-2 ln u0) cos(2 pi u1),  z[4q+1] = sqrt(-2 ln u0) sin(2 pi u1),
-    z[4q+2] = sqrt(-2 ln u2) cos(2 pi u3),  z[4q+3] = sqrt(-2 ln u2) sin(2 pi u3).
+    One Philox4x64-10 draw with counter (i * d/8 + q, hq, b, layer_id) and key
+    (seed, 0) covers dims 4q..4q+3 and d/2+4q..d/2+4q+3 of proxy i of query
+    head hq. Its four 64-bit outputs, split low word first, give eight 32-bit
+    words w0..w7 and uniforms u_k = ((w_k >> 9) + 1/2) 2^-23; Box-Muller turns
+    each pair (u_2m, u_2m+1) into sqrt(-2 ln u_2m) (cos, sin)(2 pi u_2m+1).
+    Pairs 0, 1 fill dims 4q..4q+3; pairs 2, 3 fill d/2+4q..d/2+4q+3.
     """
-    assert head_dim % 4 == 0
-    nq = head_dim // 4
+    assert head_dim % 8 == 0
+    nq = head_dim // 8
     hq, i, q = np.meshgrid(np.arange(n_q_heads, dtype=np.uint64),
                            np.arange(n_proxies, dtype=np.uint64),
                            np.arange(nq, dtype=np.uint64), indexing="ij")
     ctr = np.stack([i * np.uint64(nq) + q, hq,
                     np.full_like(q, np.uint64(b)),
                     np.full_like(q, np.uint64(layer_id))], axis=-1)
-    x = philox4x64_10(ctr, (seed & 0xFFFFFFFFFFFFFFFF, 0))
-    u = uniforms_from_bits(x)                               # [Hq, Np, d/4, 4]
-    r01 = np.sqrt(-2.0 * np.log(u[..., 0]))
-    r23 = np.sqrt(-2.0 * np.log(u[..., 2]))
-    z = np.empty(u.shape, dtype=np.float64)
-    z[..., 0] = r01 * np.cos(2.0 * np.pi * u[..., 1])
-    z[..., 1] = r01 * np.sin(2.0 * np.pi * u[..., 1])
-    z[..., 2] = r23 * np.cos(2.0 * np.pi * u[..., 3])
-    z[..., 3] = r23 * np.sin(2.0 * np.pi * u[..., 3])
-    return z.reshape(n_q_heads, n_proxies, head_dim)
+    x = philox4x64_10(ctr, (seed & 0xFFFFFFFFFFFFFFFF, 0))      # [Hq, Np, d/8, 4]
+    words = np.stack([x & _M32, x >> _S32], axis=-1).reshape(x.shape[:-1] + (8,))
+    u = uniforms_from_bits(words)                               # [Hq, Np, d/8, 8]
+    r = np.sqrt(-2.0 * np.log(u[..., 0::2]))                    # [.., 4]
+    ang = 2.0 * np.pi * u[..., 1::2]
+    zc, zs = r * np.cos(ang), r * np.sin(ang)
+    z = np.empty(u.shape, dtype=np.float64)                      # [.., 8]
+    z[..., 0::2] = zc
+    z[..., 1::2] = zs
+    out = np.empty((n_q_heads, n_proxies, head_dim), dtype=np.float64)
+    half = head_dim // 2
+    for k in range(4):
+        out[:, :, 4 * np.arange(nq) + k] = z[..., k]
+        out[:, :, half + 4 * np.arange(nq) + k] = z[..., 4 + k]
+    return out
 
 
 # ---------------------------------------------------------------------------
