@@ -127,19 +127,19 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   tmem_ld16(taddr + 16, *reinterpret_cast<float(*)[16]>(v + 16));
 }
 
-// Online (max, sum of exp2) update of one row over 32 logits v (columns
-// c0..c0+31 of the tile; columns >= nvalid are past the split and ignored).
+// Online (max, sum of exp2) update of one row over 32 logits v (columns past
+// the end of the split are set to -inf beforehand by mask_tail).
 // m is the running max of the log2-scaled logits, z the sum of exp2(x - m).
 // The max is only raised when the chunk's sum relative to it would exceed
 // 2^100 (or on the first chunk), so the common path is FFMA + EX2 + FADD; z
 // stays below 2^127 over the 32 chunks of a key split.
-__device__ __forceinline__ void softmax_chunk(float (&v)[32], int c0, int nvalid, float alpha,
-                                              float& m, float& z) {
-  if (nvalid < c0 + 32) {
+__device__ __noinline__ void mask_tail(float (&v)[32], int c0, int nvalid) {
 #pragma unroll
-    for (int j = 0; j < 32; ++j)
-      if (c0 + j >= nvalid) v[j] = -INFINITY;
-  }
+  for (int j = 0; j < 32; ++j)
+    if (c0 + j >= nvalid) v[j] = -INFINITY;
+}
+
+__device__ __forceinline__ void softmax_chunk(float (&v)[32], float alpha, float& m, float& z) {
   const float nm = -m;
   float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
 #pragma unroll
@@ -414,12 +414,23 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         if (PASS == 1) {
           const int nvalid = min(BK, x.t1 - kt);
           const uint32_t tcol = tacc + (uint32_t)(sub * 128);
+          if (nvalid == BK) {            // every tile but the last of a short split
 #pragma unroll 1
-          for (int c0 = 0; c0 < BK; c0 += 32) {
-            float v[32];
-            tmem_ld32(tcol + c0, v);
-            tmem_wait_ld();
-            softmax_chunk(v, c0, nvalid, alpha, m_run, z_run);
+            for (int c0 = 0; c0 < BK; c0 += 32) {
+              float v[32];
+              tmem_ld32(tcol + c0, v);
+              tmem_wait_ld();
+              softmax_chunk(v, alpha, m_run, z_run);
+            }
+          } else {
+#pragma unroll 1
+            for (int c0 = 0; c0 < BK; c0 += 32) {
+              float v[32];
+              tmem_ld32(tcol + c0, v);
+              tmem_wait_ld();
+              mask_tail(v, c0, nvalid);
+              softmax_chunk(v, alpha, m_run, z_run);
+            }
           }
         } else {
           const int t = kt + lrow;
