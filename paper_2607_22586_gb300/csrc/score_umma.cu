@@ -21,10 +21,14 @@
 // Softmax pass (PASS 1): stationary = 2 x 128 proxy rows as the M operand,
 //   K tile = N operand (M=128, N=128, two MMAs); the accumulator lane is a
 //   proxy row, so each thread keeps its row's running (max, sum of exp2) over
-//   the 128 keys of a tile without any cross-thread reduction. The running max
-//   is only raised when a 32-key chunk's sum would exceed 2^100 (or on the
-//   first chunk), and it is carried over from split to split of the same
-//   block, so the common path is one FFMA, one MUFU.EX2 and one FADD per logit.
+//   the 128 keys of a tile without any cross-thread reduction. Each split
+//   starts from the max of its first 32-key chunk; after that the max is only
+//   raised when a chunk's sum would exceed 2^100, so the common path is one
+//   FFMA, one MUFU.EX2 and one FADD per logit.
+// Tile j of a split goes to accumulator j mod 2 and a split's partial starts
+// afresh, so every split's results are the same whichever CTA runs it and
+// whatever it ran before: a stack of layers in one call gives the same bits
+// as the layers called one by one.
 // Mass pass (PASS 2): K tile = M operand (128 keys), stationary = up to 256
 //   proxy rows holding whole groups as the N operand; the accumulator lane is
 //   a key, so each thread sums exp2(x - c_row) over the columns of a group in
@@ -131,7 +135,7 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
 // the end of the split are set to -inf beforehand by mask_tail).
 // m is the running max of the log2-scaled logits, z the sum of exp2(x - m).
 // The max is only raised when the chunk's sum relative to it would exceed
-// 2^100 (or on the first chunk), so the common path is FFMA + EX2 + FADD; z
+// 2^100 (or while it is still -inf), so the common path is FFMA + EX2 + FADD; z
 // stays below 2^127 over the 32 chunks of a key split.
 __device__ __noinline__ void mask_tail(float (&v)[32], int c0, int nvalid) {
 #pragma unroll
@@ -172,6 +176,29 @@ __device__ __forceinline__ void softmax_chunk(float (&v)[32], float alpha, float
     }
   }
   z += zc;
+}
+
+// First chunk of a split: the reference is the chunk's own max (ALU only, so
+// the exponentials are evaluated once); z starts from this chunk's sum.
+__device__ __forceinline__ void softmax_first(const float (&v)[32], float alpha, float& m, float& z) {
+  float c0 = -INFINITY, c1 = -INFINITY;
+#pragma unroll
+  for (int j = 0; j < 32; j += 2) {
+    c0 = fmaxf(c0, v[j] * alpha);
+    c1 = fmaxf(c1, v[j + 1] * alpha);
+  }
+  m = fmaxf(c0, c1);
+  if (m == -INFINITY) return;      // every column masked: nothing to add
+  const float nm = -m;
+  float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+  for (int j = 0; j < 32; j += 4) {
+    s0 += fast_exp2(fmaf(v[j], alpha, nm));
+    s1 += fast_exp2(fmaf(v[j + 1], alpha, nm));
+    s2 += fast_exp2(fmaf(v[j + 2], alpha, nm));
+    s3 += fast_exp2(fmaf(v[j + 3], alpha, nm));
+  }
+  z = (s0 + s1) + (s2 + s3);
 }
 
 // 16 consecutive row normalisers from the warp's shared-memory copy.
@@ -321,8 +348,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      int stage = 0, buf = 0;
-      uint32_t phase = 0, bphase = 0, sphase = 0;
+      int stage = 0;
+      uint32_t phase = 0, bphase = 0, sphase = 0;   // bphase: one phase bit per accumulator
       long long prev = -1;
       uint32_t idesc = idesc_bf16_f32(128, 128);
       for (int sr = s_begin; sr < s_end; ++sr) {
@@ -338,9 +365,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           prev = key;
         }
         bool ok = true;
-        for (int kt = x.t0; kt < x.t1; kt += BK) {
+        // accumulator = parity of the tile's index within its split, so a
+        // split's tiles reach the same epilogue warpgroups whatever ran before
+        for (int kt = x.t0, j = 0; kt < x.t1; kt += BK, ++j) {
+          const int buf = j & 1;
           if (!mbar_wait(&full[stage], phase, abort_) ||
-              !mbar_wait(&tempty[buf], bphase ^ 1u, abort_)) { ok = false; break; }
+              !mbar_wait(&tempty[buf], ((bphase >> buf) & 1u) ^ 1u, abort_)) { ok = false; break; }
           fence_after();
           const uint32_t ks_base = smem_u32(ring + stage * SM::STAGE_BYTES);
           const uint32_t st_base = smem_u32(stat);
@@ -363,8 +393,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           mma_commit(&empty[stage]);
           mma_commit(&tfull[buf]);
           if (++stage == NSTAGE) { stage = 0; phase ^= 1u; }
-          buf ^= 1;
-          if (buf == 0) bphase ^= 1u;
+          bphase ^= 1u << buf;
         }
         if (!ok) break;
       }
@@ -381,17 +410,18 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     const int q = warp % 4;               // TMEM lane quarter this warp may access
     const int lrow = q * 32 + lane;       // accumulator lane: proxy row (1) / key (2)
     const float alpha = P.alpha;
-    uint32_t ntile = 0;                   // tiles seen, in the MMA's order
-    long long prev = -1, prev_blk = -1;
-    float m_run = -INFINITY;              // softmax pass: reference max of this thread's row
+    uint32_t bphase = 0;                  // one phase bit per accumulator
+    long long prev_blk = -1;
     for (int sr = s_begin; sr < s_end; ++sr) {
       const int u = sr * S.ntiles + my_tile;
       const Unit x = decode(P, S, u);
       const ReqInfo R = P.req[x.b];
       const long long key = block_key(P, S, x);
-      if (key != prev) m_run = -INFINITY;  // a new row: no reference yet
-      prev = key;
-      float z_run = 0.f;                   // sum of exp2(x - m_run) over this split
+      // softmax pass: (reference max, sum of exp2(x - max)) of this thread's
+      // row over its tiles of this split; restarted per split so that the
+      // split's partial does not depend on what the CTA ran before
+      float m_run = -INFINITY, z_run = 0.f;
+      bool first = true;
       Block blk{};
       const float* cv = cs_all + ew * SROWS;   // this warp's copy of the block's normalisers
       if (PASS == 2) {
@@ -405,10 +435,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         }
       }
       bool ok = true;
-      for (int kt = x.t0; kt < x.t1; kt += BK, ++ntile) {
-        const int buf = (int)(ntile & 1u);
+      for (int kt = x.t0, j = 0; kt < x.t1; kt += BK, ++j) {
+        const int buf = j & 1;
         if (buf != par) continue;
-        if (!mbar_wait(&tfull[buf], (ntile >> 1) & 1u, abort_)) { ok = false; break; }
+        const uint32_t ph = (bphase >> buf) & 1u;
+        bphase ^= 1u << buf;
+        if (!mbar_wait(&tfull[buf], ph, abort_)) { ok = false; break; }
         fence_after();
         const uint32_t tacc = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * ACC_STRIDE);
         if (PASS == 1) {
@@ -420,7 +452,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
               float v[32];
               tmem_ld32(tcol + c0, v);
               tmem_wait_ld();
-              softmax_chunk(v, alpha, m_run, z_run);
+              if (first) {
+                softmax_first(v, alpha, m_run, z_run);
+                first = false;
+              } else {
+                softmax_chunk(v, alpha, m_run, z_run);
+              }
             }
           } else {
 #pragma unroll 1
@@ -429,7 +466,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
               tmem_ld32(tcol + c0, v);
               tmem_wait_ld();
               mask_tail(v, c0, nvalid);
-              softmax_chunk(v, alpha, m_run, z_run);
+              if (first) {
+                softmax_first(v, alpha, m_run, z_run);
+                first = false;
+              } else {
+                softmax_chunk(v, alpha, m_run, z_run);
+              }
             }
           }
         } else {

@@ -100,8 +100,12 @@ def test_select_hyperparameters(kw):
     _check_all(wl, gpu, refs, h, what=str(kw))
 
 
-def test_multi_layer_call_matches_single_layer_calls():
-    wl = RAGGED.replace(seq_lens=(200, 333), n_visual=(190, 300), budgets=(50, 64))
+@pytest.mark.parametrize("lens", [(200, 333), (3000, 1333)])
+def test_multi_layer_call_matches_single_layer_calls(lens):
+    """Bitwise equal whether the layers run in one call or one by one; the
+    longer requests span several key splits (one with an odd tile count), so
+    the CTAs' split ranges start at different places in the two calls."""
+    wl = RAGGED.replace(seq_lens=lens, n_visual=(lens[0] - 10, lens[1] - 33), budgets=(50, 64))
     lis = [S.make_layer(wl, l) for l in range(3)]
     h = PT.hyper(n_proxies=64, n_groups=4, seed=9, layer_id=2)
     multi = PT.gpu_select(wl, lis, h)
