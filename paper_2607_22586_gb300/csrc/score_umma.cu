@@ -21,7 +21,8 @@
 // Softmax pass (PASS 1): stationary = 2 x 128 proxy rows as the M operand,
 //   K tile = N operand (M=128, N=128, two MMAs); the accumulator lane is a
 //   proxy row, so each thread keeps its row's running (max, sum of exp2) over
-//   the 128 keys of a tile without any cross-thread reduction. Each split
+//   its 64-key half of every tile without any cross-thread reduction (one
+//   partial per row, key half and split). Each split
 //   starts from the max of its first 32-key chunk; after that the max is only
 //   raised when a chunk's sum would exceed 2^100, so the common path is one
 //   FFMA, one MUFU.EX2 and one FADD per logit.
@@ -52,7 +53,7 @@ constexpr int SROWS = 256;       // stationary proxy rows per block
 constexpr int NSTAGE = 4;        // K-tile ring depth
 constexpr int NTHREADS = 576;
 constexpr int EPI_WARP0 = 2;
-constexpr int NEPI = 512;        // epilogue threads: 4 warpgroups, 2 per accumulator
+constexpr int NEPI = 512;        // epilogue threads: 4 warpgroups
 constexpr int TMEM_COLS = 512;
 constexpr int ACC_STRIDE = 256;  // TMEM columns per accumulator buffer
 
@@ -143,17 +144,29 @@ __device__ __noinline__ void mask_tail(float (&v)[32], int c0, int nvalid) {
     if (c0 + j >= nvalid) v[j] = -INFINITY;
 }
 
-__device__ __forceinline__ void softmax_chunk(float (&v)[32], float alpha, float& m, float& z) {
-  const float nm = -m;
-  float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+// Sum over 32 logits of exp2(v * alpha - m) into four interleaved partial
+// sums (column j feeds sum j mod 4), then (s0 + s1) + (s2 + s3). The scale
+// and the additions run as packed pairs.
+__device__ __forceinline__ float exp2_sum32(const float (&v)[32], uint64_t al2, float m) {
+  const uint64_t nm2 = pk2(-m, -m);
+  uint64_t s01 = 0, s23 = 0;       // the bit pattern 0 is (+0, +0)
 #pragma unroll
   for (int j = 0; j < 32; j += 4) {
-    s0 += fast_exp2(fmaf(v[j], alpha, nm));
-    s1 += fast_exp2(fmaf(v[j + 1], alpha, nm));
-    s2 += fast_exp2(fmaf(v[j + 2], alpha, nm));
-    s3 += fast_exp2(fmaf(v[j + 3], alpha, nm));
+    float y0, y1, y2, y3;
+    upk2(ffma2(pk2(v[j], v[j + 1]), al2, nm2), y0, y1);
+    upk2(ffma2(pk2(v[j + 2], v[j + 3]), al2, nm2), y2, y3);
+    s01 = fadd2(s01, pk2(fast_exp2(y0), fast_exp2(y1)));
+    s23 = fadd2(s23, pk2(fast_exp2(y2), fast_exp2(y3)));
   }
-  float zc = (s0 + s1) + (s2 + s3);
+  float s0, s1, s2, s3;
+  upk2(s01, s0, s1);
+  upk2(s23, s2, s3);
+  return (s0 + s1) + (s2 + s3);
+}
+
+__device__ __forceinline__ void softmax_chunk(float (&v)[32], float alpha, float& m, float& z) {
+  const uint64_t al2 = pk2(alpha, alpha);
+  float zc = exp2_sum32(v, al2, m);
   if (!(zc <= 1.2676506e30f)) {  // first chunk, sum above 2^100 or NaN: raise the max
     float cm = -INFINITY;
 #pragma unroll
@@ -164,15 +177,7 @@ __device__ __forceinline__ void softmax_chunk(float (&v)[32], float alpha, float
     } else {
       z *= fast_exp2(m - mn);
       m = mn;
-      s0 = s1 = s2 = s3 = 0.f;
-#pragma unroll
-      for (int j = 0; j < 32; j += 4) {
-        s0 += fast_exp2(fmaf(v[j], alpha, -mn));
-        s1 += fast_exp2(fmaf(v[j + 1], alpha, -mn));
-        s2 += fast_exp2(fmaf(v[j + 2], alpha, -mn));
-        s3 += fast_exp2(fmaf(v[j + 3], alpha, -mn));
-      }
-      zc = (s0 + s1) + (s2 + s3);
+      zc = exp2_sum32(v, al2, mn);
     }
   }
   z += zc;
@@ -189,63 +194,64 @@ __device__ __forceinline__ void softmax_first(const float (&v)[32], float alpha,
   }
   m = fmaxf(c0, c1);
   if (m == -INFINITY) return;      // every column masked: nothing to add
-  const float nm = -m;
-  float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-#pragma unroll
-  for (int j = 0; j < 32; j += 4) {
-    s0 += fast_exp2(fmaf(v[j], alpha, nm));
-    s1 += fast_exp2(fmaf(v[j + 1], alpha, nm));
-    s2 += fast_exp2(fmaf(v[j + 2], alpha, nm));
-    s3 += fast_exp2(fmaf(v[j + 3], alpha, nm));
-  }
-  z = (s0 + s1) + (s2 + s3);
+  z = exp2_sum32(v, pk2(alpha, alpha), m);
 }
 
-// 16 consecutive row normalisers from the warp's shared-memory copy.
-__device__ __forceinline__ void load_c16(const float* c, float (&cv)[16]) {
-  const float4* c4 = reinterpret_cast<const float4*>(c);
+// 16 consecutive negated row normalisers (-c) from the warp's shared-memory
+// copy, as 8 packed pairs.
+__device__ __forceinline__ void load_nc16(const float* nc, uint64_t (&ncv)[8]) {
+  const ulonglong2* c2 = reinterpret_cast<const ulonglong2*>(nc);
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    const float4 t = c4[i];
-    cv[4 * i] = t.x; cv[4 * i + 1] = t.y; cv[4 * i + 2] = t.z; cv[4 * i + 3] = t.w;
+    const ulonglong2 t = c2[i];
+    ncv[2 * i] = t.x; ncv[2 * i + 1] = t.y;
   }
 }
 
-__device__ __forceinline__ void mass_chunk(const float (&v)[16], const float (&cv)[16],
-                                           float alpha, float (&a)[4]) {
+// a01 += (e_j, e_j+1), a23 += (e_j+2, e_j+3) over 16 columns, e_j =
+// exp2(v_j * alpha - c_j): column j feeds partial sum j mod 4.
+__device__ __forceinline__ void mass_chunk(const float (&v)[16], const uint64_t (&ncv)[8],
+                                           uint64_t al2, uint64_t& a01, uint64_t& a23) {
 #pragma unroll
   for (int j = 0; j < 16; j += 4) {
-    a[0] += fast_exp2(fmaf(v[j], alpha, -cv[j]));
-    a[1] += fast_exp2(fmaf(v[j + 1], alpha, -cv[j + 1]));
-    a[2] += fast_exp2(fmaf(v[j + 2], alpha, -cv[j + 2]));
-    a[3] += fast_exp2(fmaf(v[j + 3], alpha, -cv[j + 3]));
+    float y0, y1, y2, y3;
+    upk2(ffma2(pk2(v[j], v[j + 1]), al2, ncv[j / 2]), y0, y1);
+    upk2(ffma2(pk2(v[j + 2], v[j + 3]), al2, ncv[j / 2 + 1]), y2, y3);
+    a01 = fadd2(a01, pk2(fast_exp2(y0), fast_exp2(y1)));
+    a23 = fadd2(a23, pk2(fast_exp2(y2), fast_exp2(y3)));
   }
 }
 
 // Sum over the ncols (multiple of 16) accumulator columns of one group:
 // sum_j exp2(acc_j * alpha - c_j), four partial sums added in a fixed order.
-// c points at the warp's shared-memory copy of the block's normalisers.
-__device__ __forceinline__ float group_sum(uint32_t tcol, const float* c, int ncols, float alpha) {
-  float a[4] = {0.f, 0.f, 0.f, 0.f};
+// nc points at the warp's shared-memory copy of the block's negated normalisers.
+__device__ __forceinline__ float group_sum(uint32_t tcol, const float* nc, int ncols, float alpha) {
+  const uint64_t al2 = pk2(alpha, alpha);
+  uint64_t a01 = 0, a23 = 0;       // (+0, +0)
   int cc = 0;
 #pragma unroll 1
   for (; cc + 32 <= ncols; cc += 32) {
-    float v[32], cv[16];
+    float v[32];
+    uint64_t ncv[8];
     tmem_ld32(tcol + cc, v);
-    load_c16(c + cc, cv);
+    load_nc16(nc + cc, ncv);
     tmem_wait_ld();
-    mass_chunk(*reinterpret_cast<float(*)[16]>(v), cv, alpha, a);
-    load_c16(c + cc + 16, cv);
-    mass_chunk(*reinterpret_cast<float(*)[16]>(v + 16), cv, alpha, a);
+    mass_chunk(*reinterpret_cast<float(*)[16]>(v), ncv, al2, a01, a23);
+    load_nc16(nc + cc + 16, ncv);
+    mass_chunk(*reinterpret_cast<float(*)[16]>(v + 16), ncv, al2, a01, a23);
   }
   if (cc < ncols) {
-    float v[16], cv[16];
+    float v[16];
+    uint64_t ncv[8];
     tmem_ld16(tcol + cc, v);
-    load_c16(c + cc, cv);
+    load_nc16(nc + cc, ncv);
     tmem_wait_ld();
-    mass_chunk(v, cv, alpha, a);
+    mass_chunk(v, ncv, al2, a01, a23);
   }
-  return (a[0] + a[1]) + (a[2] + a[3]);
+  float a0, a1, a2, a3;
+  upk2(a01, a0, a1);
+  upk2(a23, a2, a3);
+  return (a0 + a1) + (a2 + a3);
 }
 
 template <int PASS, int D>
@@ -288,7 +294,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     mbar_init(&sempty, 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(&tfull[i], 1);
-      mbar_init(&tempty[i], NEPI / 2);
+      mbar_init(&tempty[i], PASS == 1 ? NEPI : NEPI / 2);   // drained by all / by a pair
     }
     fence_barrier_init();
     prefetch_tmap(&kmap);
@@ -400,13 +406,16 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    // Warpgroups 0,1 drain accumulator 0, warpgroups 2,3 accumulator 1, so
-    // each warpgroup takes every other key tile. In the softmax pass the
-    // two warpgroups of a pair own the two 128-row M tiles; in the mass pass
-    // they split the groups of the stationary block.
+    // Softmax pass: all four warpgroups drain every tile (warpgroup g takes
+    // M tile g & 1 and the 64-key half g >> 1), so while the CTA works on one
+    // accumulator the MMAs fill the other. Mass pass: warpgroups 0,1 drain
+    // accumulator 0 and 2,3 accumulator 1 (every other key tile), the two
+    // warpgroups of a pair splitting the groups of the stationary block.
+    // Either way every accumulator has a fixed set of consumers that waits
+    // for each of its phases in turn.
     const int ew = warp - EPI_WARP0;      // 0..15
     const int wg = ew / 4;                // warpgroup 0..3
-    const int par = wg >> 1, sub = wg & 1;
+    const int par = wg >> 1, sub = wg & 1;  // par: accumulator (mass) / key half (softmax)
     const int q = warp % 4;               // TMEM lane quarter this warp may access
     const int lrow = q * 32 + lane;       // accumulator lane: proxy row (1) / key (2)
     const float alpha = P.alpha;
@@ -423,13 +432,13 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       float m_run = -INFINITY, z_run = 0.f;
       bool first = true;
       Block blk{};
-      const float* cv = cs_all + ew * SROWS;   // this warp's copy of the block's normalisers
+      const float* cv = cs_all + ew * SROWS;   // this warp's copy of the block's negated normalisers
       if (PASS == 2) {
         blk = mass_block(P, S, x.tile);
         if (key != prev_blk) {
           const float* src = bf.cvals + (((size_t)x.l * P.B + x.b) * P.Hkv + x.h) * P.Prows_pad + blk.row0;
           __syncwarp();
-          for (int i = lane; i < blk.rows; i += 32) cs_all[ew * SROWS + i] = src[i];
+          for (int i = lane; i < blk.rows; i += 32) cs_all[ew * SROWS + i] = -src[i];
           __syncwarp();
           prev_blk = key;
         }
@@ -437,18 +446,19 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       bool ok = true;
       for (int kt = x.t0, j = 0; kt < x.t1; kt += BK, ++j) {
         const int buf = j & 1;
-        if (buf != par) continue;
+        if (PASS == 2 && buf != par) continue;
         const uint32_t ph = (bphase >> buf) & 1u;
         bphase ^= 1u << buf;
         if (!mbar_wait(&tfull[buf], ph, abort_)) { ok = false; break; }
         fence_after();
         const uint32_t tacc = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * ACC_STRIDE);
         if (PASS == 1) {
-          const int nvalid = min(BK, x.t1 - kt);
-          const uint32_t tcol = tacc + (uint32_t)(sub * 128);
-          if (nvalid == BK) {            // every tile but the last of a short split
+          const int c_lo = par * (BK / 2);           // this warpgroup's key half
+          const int nvalid = min(BK, x.t1 - kt) - c_lo;
+          const uint32_t tcol = tacc + (uint32_t)(sub * 128 + c_lo);
+          if (nvalid >= BK / 2) {        // every tile but the last of a short split
 #pragma unroll 1
-            for (int c0 = 0; c0 < BK; c0 += 32) {
+            for (int c0 = 0; c0 < BK / 2; c0 += 32) {
               float v[32];
               tmem_ld32(tcol + c0, v);
               tmem_wait_ld();
@@ -461,7 +471,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             }
           } else {
 #pragma unroll 1
-            for (int c0 = 0; c0 < BK; c0 += 32) {
+            for (int c0 = 0; c0 < BK / 2; c0 += 32) {
               float v[32];
               tmem_ld32(tcol + c0, v);
               tmem_wait_ld();

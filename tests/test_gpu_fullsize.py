@@ -70,18 +70,38 @@ def _check_units(wl, gpu, lis, layer_ids, h, units, proxies=None):
         PT.check_gather(g, wl, li_pos, lo, int(outs[b]), keep, hi - lo, 1)
 
 
-def test_long_context_stack_full_size():
-    """28 layers x 32768 tokens (4 images + text), all layers in one call;
-    oracle on layers 0, 14, 27 x all KV heads."""
+@pytest.fixture(scope="module")
+def stack32k():
+    """The 28-layer x 32768-token stack with given proxies, generated once."""
     wl = S.WORKLOADS["qwen7b-28l-32k"]
     ids = list(range(wl.n_layers))
     lis = _layers(wl, ids)
     h = PT.hyper()
     prox = np.stack([S.make_proxies(wl, h["n_proxies"], l) for l in ids])
+    return wl, ids, lis, h, prox
+
+
+def test_long_context_stack_full_size(stack32k):
+    """28 layers x 32768 tokens (4 images + text), all layers in one call;
+    oracle on layers 0, 14, 27 x all KV heads."""
+    wl, ids, lis, h, prox = stack32k
     gpu = PT.gpu_select(wl, lis, h, proxies=prox)
     assert gpu["score_path"] == 1
     units = [(l, 0, kvh) for l in (0, 14, 27) for kvh in range(wl.n_kv_heads)]
     _check_units(wl, gpu, lis, ids, h, units, proxies=prox)
+
+
+def test_long_context_stack_repeatable(stack32k):
+    """The full-size call twice gives the same bits (each split's partials do
+    not depend on CTA timing), and layer 0 alone gives those of the stack."""
+    wl, ids, lis, h, prox = stack32k
+    a = PT.gpu_select(wl, lis, h, proxies=prox)
+    b = PT.gpu_select(wl, lis, h, proxies=prox)
+    for key in ("group_mass", "anchor", "idx", "out_k"):
+        np.testing.assert_array_equal(a[key], b[key], err_msg=key)
+    one = PT.gpu_select(wl, [lis[0]], h, proxies=prox[:1])
+    for key in ("group_mass", "anchor", "idx"):
+        np.testing.assert_array_equal(a[key][0], one[key][0], err_msg=key)
 
 
 def test_long_context_stack_sampled_proxies():
