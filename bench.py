@@ -208,6 +208,50 @@ def score_traffic(wl, args, kernel):
     return t.get(kernel)
 
 
+class Ranks:
+    """One process per GPU, as torchrun starts them (RANK, WORLD_SIZE,
+    LOCAL_RANK, MASTER_ADDR / MASTER_PORT from the environment). With more
+    than one rank a process group over ``backend`` is opened; every rank runs
+    its own replica of the workload (no data-path collective), and only the
+    timing uses the group: barriers around the timed region and the maximum of
+    the per-rank times."""
+
+    def __init__(self, backend: str):
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.local = int(os.environ.get("LOCAL_RANK", "0"))
+        self.dist = None
+        if self.world > 1:
+            import torch.distributed as dist
+            dist.init_process_group(backend)
+            self.dist = dist
+
+    def barrier(self):
+        if self.dist:
+            self.dist.barrier()
+
+    def max(self, x: float, device=None) -> float:
+        """Maximum of x over the ranks (x itself with one rank)."""
+        if not self.dist:
+            return float(x)
+        import torch
+        t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+        self.dist.all_reduce(t, op=self.dist.ReduceOp.MAX)
+        return float(t.item())
+
+    def close(self):
+        if self.dist:
+            self.dist.barrier()
+            self.dist.destroy_process_group()
+            self.dist = None
+
+
+def job_value(tokens_per_rank: float, world: int, ms_max: float) -> float:
+    """Whole-job throughput: the tokens every rank processed in one step over
+    the slowest rank's step time."""
+    return tokens_per_rank * world / (ms_max * 1e-3)
+
+
 def run_reference(args, wl):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -245,16 +289,9 @@ def run_gpu(args, wl):
     import paper_2607_22586_gb300 as M
     from paper_2607_22586_gb300 import _lib as LB
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    dist = None
-    if world > 1:
-        import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl")
-    else:
-        torch.cuda.set_device(0)
+    torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+    ranks = Ranks("nccl")
+    world, rank = ranks.world, ranks.rank
     dev = torch.device("cuda", torch.cuda.current_device())
     hyper = hyper_for(args, wl)
     peaks, peak_src = read_peaks()
@@ -304,23 +341,17 @@ def run_gpu(args, wl):
     clocks.start()
     time.sleep(0.3)
     torch.cuda.synchronize()
-    if dist:
-        dist.barrier()
+    ranks.barrier()
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     t_start.record(stream)
     for k in range(args.steps):
         step(dbgs[k])
     t_end.record(stream)
     torch.cuda.synchronize()
-    if dist:
-        dist.barrier()
+    ranks.barrier()
     clk = clocks.stop()
     M.check(M.mmshift_poll_status(ws, stream), "timed status")
-    ms = t_start.elapsed_time(t_end) / args.steps
-    if dist:
-        tt = torch.tensor([ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms = ranks.max(t_start.elapsed_time(t_end) / args.steps, dev)
     stage_ms = {name: statistics.mean(ev[i].elapsed_time(ev[i + 1]) for ev in stage_ev)
                 for i, name in enumerate(LB.STAGES)}
     launches = dbgs[0].launches * args.steps
@@ -331,8 +362,7 @@ def run_gpu(args, wl):
     ov_h = torch.empty_like(ok_h, pin_memory=True)
     e_steps = max(1, args.steps)
     torch.cuda.synchronize()
-    if dist:
-        dist.barrier()
+    ranks.barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for _ in range(e_steps):
@@ -345,17 +375,13 @@ def run_gpu(args, wl):
         ov_h.copy_(out_v, non_blocking=True)
     e1.record(stream)
     torch.cuda.synchronize()
-    e_ms = e0.elapsed_time(e1) / e_steps
-    if dist:
-        tt = torch.tensor([e_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e_ms = float(tt.item())
+    e_ms = ranks.max(e0.elapsed_time(e1) / e_steps, dev)
     h2d = sum(t.numel() * t.element_size() for t in (K_pin, V_pin, Q_pin))
     d2h = sum(t.numel() * t.element_size() for t in (idx_h, ok_h, ov_h))
 
     bytes_step, k_read, pass_flops = algorithmic(wl, hyper)
-    tokens_layer = T * L * world
-    value = tokens_layer / (ms * 1e-3)
+    tokens_layer = T * L * world          # metric unit: tokens per second per layer
+    value = job_value(T * L, world, ms)
     hbm_frac = bytes_step / (ms * 1e-3) / (peaks["hbm_gbs"] * 1e9)
 
     # dominant stage and its roofline
@@ -407,7 +433,7 @@ def run_gpu(args, wl):
         "stage_ms": stage_ms,
         "roofline": roof,
         "cpu_baseline": cpu,
-        "e2e": {"value": tokens_layer / (e_ms * 1e-3), "unit": UNIT, "ms_per_step": e_ms,
+        "e2e": {"value": job_value(T * L, world, e_ms), "unit": UNIT, "ms_per_step": e_ms,
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "clocks": clk,
         "gpu_launches": launches,
@@ -415,9 +441,7 @@ def run_gpu(args, wl):
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
-    if dist:
-        dist.barrier()
-        dist.destroy_process_group()
+    ranks.close()
     return 0
 
 
