@@ -45,11 +45,11 @@ SFU_EX2_PER_SM_CLK = 32          # MUFU.EX2 lanes per SM per clock on GB300 (mea
 
 # DRAM traffic (read + write) of the two scoring kernels per launch of the
 # default workload, from one ncu capture of a 4-layer slice scaled by 7 to the
-# 28 layers (traffic grows with the layers; profiles/kernels_qwen7b-32k-4layers
-# _full-set.md). It describes the score_umma.cu it was measured on only.
-SCORE_TRAFFIC = {"source_sha256_16": "88d5d81df09ba7fb", "workload": "qwen7b-28l-32k",
-                 "proxies": "paper", "softmax_pass": 7 * (157.078784e6 + 19.625984e6),
-                 "mass_pass": 7 * (156.657408e6 + 46.612224e6)}
+# 28 layers (traffic grows with the layers). It describes only the
+# score_umma.cu it was measured on (checked by hash).
+SCORE_TRAFFIC = {"source_sha256_16": "c2be9d2f4efd6f44", "workload": "qwen7b-28l-32k",
+                 "proxies": "paper", "softmax_pass": 7 * (157.129984e6 + 19.448576e6),
+                 "mass_pass": 7 * (156.619264e6 + 46.906624e6)}
 UNIT = "tokens/s/layer"
 SM_COUNT = 152
 FP32_LANES_PER_SM = 128
