@@ -71,9 +71,40 @@ struct KeySrc {
   }
 };
 
-__device__ __forceinline__ unsigned long long fx_weight(uint32_t key, int shift) {
+// Weight of a key in 2^-shift units: x * 2^shift is exact (a power-of-two
+// scale of a finite value well inside the float range), then rounded to an
+// integer.
+__device__ __forceinline__ float pow2f(int shift) { return __int_as_float((127 + shift) << 23); }
+__device__ __forceinline__ unsigned long long fx_weight(uint32_t key, float scale) {
   const float x = fmaxf(key_value(key), 0.f);
-  return __float2ull_rn(ldexpf(x, shift));
+  return __float2ull_rn(x * scale);
+}
+
+// Add a 64-bit weight to a histogram bin held as two 32-bit words (low,
+// high): the carry out of the low word is detected from the atomic's return.
+__device__ __forceinline__ void add_weight(uint32_t* lo_w, uint32_t* hi_w, unsigned long long wt) {
+  const uint32_t lo = (uint32_t)wt;
+  uint32_t hi = (uint32_t)(wt >> 32);
+  if (lo) {
+    const uint32_t old = atomicAdd(lo_w, lo);
+    hi += (old + lo < old) ? 1u : 0u;
+  }
+  if (hi) atomicAdd(hi_w, hi);
+}
+
+// 32 x 32 bit-matrix transpose across a warp: on entry lane i holds row i
+// (bit j = element (i, j)), on return lane j holds column j (bit i = element
+// (i, j)). Five rounds swap the off-diagonal s x s blocks (s = 16 .. 1)
+// between lanes i and i ^ s.
+__device__ __forceinline__ uint32_t warp_transpose32(uint32_t x) {
+  const int lane = threadIdx.x & 31;
+  uint32_t m = 0x0000FFFFu;
+#pragma unroll
+  for (int s = 16; s > 0; s >>= 1, m ^= m << s) {
+    const uint32_t y = __shfl_xor_sync(0xffffffffu, x, s);
+    x = (lane & s) ? ((x & ~m) | ((y >> s) & m)) : ((x & m) | ((y & m) << s));
+  }
+  return x;
 }
 
 // Block-wide exclusive scan of one unsigned per warp (warp totals in S.wcnt).
@@ -107,6 +138,7 @@ __device__ __forceinline__ void digit_histogram(const KeySrc& get, int n, uint32
   __syncwarp();
   unsigned long long tot = 0;
   uint32_t kmax = 0;
+  const float scale = pow2f(shift);
   constexpr int U = 8;  // independent loads in flight per thread
   for (int base = 0; base < n; base += U * NTH) {
     uint32_t kk[U];
@@ -125,15 +157,9 @@ __device__ __forceinline__ void digit_histogram(const KeySrc& get, int n, uint32
         const uint32_t d = (k >> sh) & dmask;
         atomicAdd(&hn[d], 1u);
         if (WEIGHTED) {
-          const unsigned long long wt = fx_weight(k, shift);
+          const unsigned long long wt = fx_weight(k, scale);
           if (first) { tot += wt; kmax = max(kmax, k); }
-          const uint32_t lo = (uint32_t)wt;
-          uint32_t hi = (uint32_t)(wt >> 32);
-          if (lo) {
-            const uint32_t old = atomicAdd(&hlo[d], lo);
-            hi += (old + lo < old) ? 1u : 0u;   // carry out of the low word
-          }
-          if (hi) atomicAdd(&hhi[d], hi);
+          add_weight(&hlo[d], &hhi[d], wt);
         }
       }
     }
@@ -277,7 +303,7 @@ __global__ void __launch_bounds__(NTC, 4) cover_kernel(Problem P, Buffers bf) {
   const unsigned n_theta = S.n_theta;
   const unsigned long long target =
       min(S.total, (unsigned long long)ceil((double)P.tau * (double)S.total));
-  const unsigned long long wth = fx_weight(theta, shift);
+  const unsigned long long wth = fx_weight(theta, pow2f(shift));
   const unsigned long long need_w = target > S.cum_w ? target - S.cum_w : 0ull;
   unsigned n_tie = 1;
   if (need_w > 0 && wth > 0) n_tie = (unsigned)((need_w + wth - 1) / wth);
@@ -347,34 +373,56 @@ __global__ void __launch_bounds__(NT, 1) topk_kernel(Problem P, Buffers bf, int3
   if (!from_scores) {
     const float* an = bf.anchor + hrow;
     const uint32_t* bw = bf.bits + ((size_t)l * P.Hkv + h) * P.G * P.total_words + R.word_off;
-    // each warp takes 32 consecutive keys at a time
-    for (int base = w * 32; base < n; base += NT) {
-      const int i = base + lane;
-      float s;
+    // each warp takes 32 consecutive keys at a time, UB chunks of them with
+    // their loads in flight together
+    constexpr int UB = 8;
+    for (int base0 = w * 32; base0 < n; base0 += UB * NT) {
+      float sv[UB];
       if (P.mode == MMSHIFT_SCORE_VOTE) {
-        // lane g holds the coverage word of group g for these 32 keys; the
-        // vote of key base+j is the number of lanes whose bit j is set
-        unsigned vote = 0;
+        // lane g holds the coverage word of group g for a chunk of 32 keys;
+        // after the transpose lane j holds the bits of key base+j over the
+        // groups, and its vote is their count
+        unsigned vote[UB];
+        float av[UB];
+#pragma unroll
+        for (int u = 0; u < UB; ++u) {
+          vote[u] = 0;
+          const int i = base0 + u * NT + lane;
+          av[u] = i < n ? __ldg(an + i) : 0.f;
+        }
         for (int g0 = 0; g0 < P.G; g0 += 32) {
           const int g = g0 + lane;
-          const uint32_t word = g < P.G ? bw[(size_t)g * P.total_words + (base >> 5)] : 0u;
+          uint32_t word[UB];
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const unsigned c = __popc(__ballot_sync(0xffffffffu, (word >> j) & 1u));
-            if (lane == j) vote += c;
+          for (int u = 0; u < UB; ++u) {
+            const int base = base0 + u * NT;
+            word[u] = (g < P.G && base < n) ? __ldg(bw + (size_t)g * P.total_words + (base >> 5)) : 0u;
+          }
+#pragma unroll
+          for (int u = 0; u < UB; ++u) vote[u] += __popc(warp_transpose32(word[u]));
+        }
+#pragma unroll
+        for (int u = 0; u < UB; ++u)
+          sv[u] = __fadd_rn((float)vote[u], __fmul_rn(P.lambda, av[u]));  // no contraction
+      } else {
+#pragma unroll
+        for (int u = 0; u < UB; ++u) sv[u] = 0.f;
+        for (int g = 0; g < P.G; ++g) {
+          const float* gm = bf.gmass + (((size_t)l * P.Hkv + h) * P.G + g) * P.total_T + R.tok_off;
+#pragma unroll
+          for (int u = 0; u < UB; ++u) {
+            const int i = base0 + u * NT + lane;
+            if (i < n) sv[u] += __ldg(gm + i);
           }
         }
-        s = i < n ? __fadd_rn((float)vote, __fmul_rn(P.lambda, an[i])) : 0.f;  // no contraction
-      } else {
-        float ms = 0.f;
-        if (i < n)
-          for (int g = 0; g < P.G; ++g)
-            ms += bf.gmass[(((size_t)l * P.Hkv + h) * P.G + g) * P.total_T + R.tok_off + i];
-        s = ms;
       }
-      if (i < n) {
-        sc[i] = s;
-        if (staged) keys_sm[i] = nonneg_key(s);
+#pragma unroll
+      for (int u = 0; u < UB; ++u) {
+        const int i = base0 + u * NT + lane;
+        if (i < n) {
+          sc[i] = sv[u];
+          if (staged) keys_sm[i] = nonneg_key(sv[u]);
+        }
       }
     }
   } else if (staged) {
