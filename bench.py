@@ -47,9 +47,9 @@ SFU_EX2_PER_SM_CLK = 32          # MUFU.EX2 lanes per SM per clock on GB300 (mea
 # default workload, from one ncu capture of a 4-layer slice scaled by 7 to the
 # 28 layers (traffic grows with the layers). It describes only the
 # score_umma.cu it was measured on (checked by hash).
-SCORE_TRAFFIC = {"source_sha256_16": "c2be9d2f4efd6f44", "workload": "qwen7b-28l-32k",
-                 "proxies": "paper", "softmax_pass": 7 * (157.129984e6 + 19.448576e6),
-                 "mass_pass": 7 * (156.619264e6 + 46.906624e6)}
+SCORE_TRAFFIC = {"source_sha256_16": "dc3a01adad94c3e9", "workload": "qwen7b-28l-32k",
+                 "proxies": "paper", "softmax_pass": 7 * (154.181632e6 + 44.690176e6),
+                 "mass_pass": 7 * (156.648704e6 + 46.562816e6)}
 UNIT = "tokens/s/layer"
 SM_COUNT = 152
 FP32_LANES_PER_SM = 128
@@ -361,11 +361,8 @@ def run_gpu(args, wl):
     ok_h = torch.empty(out_k.shape, dtype=out_k.dtype, pin_memory=True)
     ov_h = torch.empty_like(ok_h, pin_memory=True)
     e_steps = max(1, args.steps)
-    torch.cuda.synchronize()
-    ranks.barrier()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(e_steps):
+
+    def e2e_step():
         K.copy_(K_pin, non_blocking=True)
         V.copy_(V_pin, non_blocking=True)
         Q.copy_(Q_pin, non_blocking=True)
@@ -373,6 +370,14 @@ def run_gpu(args, wl):
         idx_h.copy_(out_idx, non_blocking=True)
         ok_h.copy_(out_k, non_blocking=True)
         ov_h.copy_(out_v, non_blocking=True)
+
+    e2e_step()                    # untimed warm-up of the pinned host buffers
+    torch.cuda.synchronize()
+    ranks.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(e_steps):
+        e2e_step()
     e1.record(stream)
     torch.cuda.synchronize()
     e_ms = ranks.max(e0.elapsed_time(e1) / e_steps, dev)

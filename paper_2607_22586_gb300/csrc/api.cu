@@ -138,7 +138,7 @@ Layout layout_of(const Problem& P) {
   size_t o = 0;
   w.status = o; o += 256;
   w.packed = o; o += align256(L * P.B * P.Hkv * (size_t)P.Prows_pad * P.d * esz);
-  w.part = o;   o += align256(L * P.Hkv * (size_t)P.total_splits * 2 * P.Prows_pad * sizeof(float2));
+  w.part = o;   o += align256(L * P.Hkv * (size_t)P.total_splits * kUmmaPartSlots * P.Prows_pad * sizeof(float2));
   w.cvals = o;  o += align256(L * P.B * P.Hkv * (size_t)P.Prows_pad * sizeof(float));
   w.gmass = o;  o += align256(L * P.Hkv * (size_t)P.G * P.total_T * sizeof(float));
   w.anchor = o; o += align256(L * P.Hkv * (size_t)P.total_T * sizeof(float));
@@ -296,7 +296,7 @@ mmshift_status mmshift_proxy_mass(const mmshift_shape* s, const void* K, const v
   if (st != MMSHIFT_OK) return st;
   if (!p || !K || !Qwin || !anchor || (P.G && !group_mass)) return MMSHIFT_ERR_INVALID_ARG;
   P.use_umma = choose_umma(P, K);
-  P.part_slots = P.use_umma ? 2 : 1;
+  P.part_slots = P.use_umma ? kUmmaPartSlots : 1;
   Buffers bf;
   if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
   bf.proxies_in = proxies;
@@ -365,7 +365,7 @@ mmshift_status mmshift_select(const mmshift_shape* s, const void* K, const void*
   if (st != MMSHIFT_OK) return st;
   if (!p || !K || !V || !Qwin || !out_idx || !out_K || !out_V) return MMSHIFT_ERR_INVALID_ARG;
   P.use_umma = choose_umma(P, K);
-  P.part_slots = P.use_umma ? 2 : 1;
+  P.part_slots = P.use_umma ? kUmmaPartSlots : 1;
   Buffers bf;
   if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
   bf.proxies_in = proxies_in;

@@ -12,6 +12,7 @@ namespace mmshift {
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr int kChunk = 16;       // proxy rows per packing chunk (one group id)
 constexpr int kRowTile = 256;    // proxy rows are padded to a multiple of this
+constexpr int kUmmaPartSlots = 4; // softmax partials per (row, split) of the tensor-core pass
 
 // Status bits the kernels OR into the workspace status word.
 enum : int {
@@ -39,6 +40,7 @@ struct Problem {
   int32_t anchor_rows; // roundup(r, 16)
   int32_t Prows;       // n_group_rows + anchor_rows
   int32_t Prows_pad;   // roundup(Prows, kRowTile)
+  int32_t part_slots;  // softmax partials per (row, key split): 1 (CUDA cores) or kUmmaPartSlots
   int32_t total_T, R, total_words, total_splits, split_len;
   int64_t ls_kv, ls_q;
   float scale, alpha, gamma, tau, lambda;
@@ -48,7 +50,6 @@ struct Problem {
   float rope_theta;
   int32_t rope_off;
   int32_t use_umma;    // steps 2-4 on the tensor cores (set per call)
-  int32_t part_slots;  // softmax partials per (row, key split): 1 (CUDA cores) or 2
   ReqInfo req[MMSHIFT_MAX_BATCH];
 };
 
@@ -108,6 +109,15 @@ __device__ __forceinline__ float fast_exp2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+// (m, z) += (m2, z2) for partial softmax normalisers: the sum of exp2(x - m)
+// over the union, relative to the larger reference max.
+__device__ __forceinline__ void merge_ms(float& m, float& z, float m2, float z2) {
+  const float mn = fmaxf(m, m2);
+  if (mn == -INFINITY) return;
+  z = z * fast_exp2(m - mn) + z2 * fast_exp2(m2 - mn);
+  m = mn;
 }
 
 __device__ __forceinline__ void set_status(int* status, int bit) {

@@ -51,12 +51,6 @@ __device__ __forceinline__ void tile_dot(const float* A, const float* Bm, int ty
   }
 }
 
-__device__ __forceinline__ void merge_ms(float& m, float& z, float m2, float z2) {
-  const float mn = fmaxf(m, m2);
-  if (mn == -INFINITY) return;
-  z = z * fast_exp2(m - mn) + z2 * fast_exp2(m2 - mn);
-  m = mn;
-}
 
 template <typename T, int D>
 __global__ void __launch_bounds__(256) pass1_simt(Problem P, Buffers bf, const T* K) {

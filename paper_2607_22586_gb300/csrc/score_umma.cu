@@ -1,39 +1,32 @@
 // Steps 2-4 on the 5th-generation tensor cores (tcgen05 + TMA + TMEM), bf16:
 // proxy logits, row softmax over the whole prompt and group-mass aggregation
-// (Section 3.2.2; Appendix B).
-//
-// Both passes are one persistent, warp-specialised kernel (one CTA per SM):
-//   warp 0      TMA producer: a stationary block of up to 256 packed proxy rows
-//               (reloaded only when the (layer, request, KV head, block) of
-//               the work unit changes) and a 4-stage ring of 128-key K tiles;
-//   warp 1      TMEM allocator and MMA issuer (one thread): d/16 tcgen05.mma
-//               of K = 16 per key tile into one of two TMEM accumulators;
-//   warps 2-17  epilogue (four warpgroups, two per TMEM accumulator):
-//               tcgen05.ld of the accumulator, exp2 and reductions in
-//               registers, outputs to global memory.
+// (Section 3.2.2; Appendix B). Two persistent, warp-specialised kernels of
+// 576 threads, one CTA per SM:
+//   warp 0      TMA producer (stationary proxy rows, a ring of K tiles);
+//   warp 1      TMEM allocator and MMA issuer (one thread);
+//   warps 2-17  epilogue (four warpgroups): tcgen05.ld of the accumulators,
+//               exp2 and reductions in registers, outputs to global memory.
 // Work units are (layer, request, KV head, key split of 1024 keys, proxy
-// block). Teams of one CTA per proxy block walk contiguous ranges of key
-// splits, so the team's CTAs read each K tile together (DRAM once, then L2)
-// and a CTA's stationary block changes only with the (layer, request, head).
-// The split boundaries (and so the merge order of the softmax partials) are
-// those of the CUDA-core path.
+// block). Teams of one CTA (softmax: one CTA pair) per proxy block walk
+// contiguous ranges of key splits, so the team reads each K tile together
+// (DRAM once, then L2) and a stationary block changes only with the (layer,
+// request, head). The split boundaries (and so the merge order of the
+// softmax partials) are those of the CUDA-core path.
 //
-// Softmax pass (PASS 1): stationary = 2 x 128 proxy rows as the M operand,
-//   K tile = N operand (M=128, N=128, two MMAs); the accumulator lane is a
-//   proxy row, so each thread keeps its row's running (max, sum of exp2) over
-//   its 64-key half of every tile without any cross-thread reduction (one
-//   partial per row, key half and split). Each split
-//   starts from the max of its first 32-key chunk; after that the max is only
-//   raised when a chunk's sum would exceed 2^100, so the common path is one
-//   FFMA, one MUFU.EX2 and one FADD per logit.
-// Tile j of a split goes to accumulator j mod 2 and a split's partial starts
-// afresh, so every split's results are the same whichever CTA runs it and
-// whatever it ran before: a stack of layers in one call gives the same bits
-// as the layers called one by one.
-// Mass pass (PASS 2): K tile = M operand (128 keys), stationary = up to 256
-//   proxy rows holding whole groups as the N operand; the accumulator lane is
-//   a key, so each thread sums exp2(x - c_row) over the columns of a group in
-//   registers and writes one group mass per key (coalesced along keys).
+// Softmax pass (softmax_pair_kernel): CTA pairs and 2-SM MMAs, below. The
+//   accumulator lane is a proxy row, so each thread keeps its row's running
+//   (max, sum of exp2) without any cross-thread reduction. Each split starts
+//   from the max of its first 32-key chunk; after that the max is only raised
+//   when a chunk's sum would exceed 2^100, so the common path is one FFMA, one
+//   MUFU.EX2 and one FADD per logit (packed in pairs). Every split's partials
+//   start afresh and land in fixed slots, so a split's results are the same
+//   whichever CTA runs it: a stack of layers in one call gives the same bits
+//   as the layers called one by one.
+// Mass pass (mass_umma_kernel): K tile = M operand (128 keys), stationary =
+//   up to 256 proxy rows holding whole groups as the N operand; the
+//   accumulator lane is a key, so each thread sums exp2(x - c_row) over the
+//   columns of a group in registers and writes one group mass per key
+//   (coalesced along keys).
 // Every wait is bounded; a CTA that gives up raises the timeout status bit,
 // stops issuing work and still frees its TMEM.
 #include <cudaTypedefs.h>
@@ -254,9 +247,9 @@ __device__ __forceinline__ float group_sum(uint32_t tcol, const float* nc, int n
   return (a0 + a1) + (a2 + a3);
 }
 
-template <int PASS, int D>
+template <int D>
 __global__ void __launch_bounds__(NTHREADS, 1)
-    score_umma_kernel(const __grid_constant__ CUtensorMap kmap,
+    mass_umma_kernel(const __grid_constant__ CUtensorMap kmap,
                       const __grid_constant__ CUtensorMap pmap, const __grid_constant__ Problem P,
                       const __grid_constant__ Sched S, Buffers bf) {
   using SM = Smem<D>;
@@ -294,7 +287,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     mbar_init(&sempty, 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(&tfull[i], 1);
-      mbar_init(&tempty[i], PASS == 1 ? NEPI : NEPI / 2);   // drained by all / by a pair
+      mbar_init(&tempty[i], NEPI / 2);   // drained by a pair of warpgroups
     }
     fence_barrier_init();
     prefetch_tmap(&kmap);
@@ -321,15 +314,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         const long long key = block_key(P, S, x);
         if (key != prev) {
           if (!mbar_wait(&sempty, sphase ^ 1u, abort_)) break;
-          int row0, rows;
-          if (PASS == 1) {
-            row0 = x.tile * SROWS;
-            rows = SROWS;
-          } else {
-            const Block k = mass_block(P, S, x.tile);
-            row0 = k.row0;
-            rows = k.rows;
-          }
+          const Block k = mass_block(P, S, x.tile);
+          const int row0 = k.row0, rows = k.rows;
           mbar_expect_tx(&sfull, (uint32_t)(rows * D * 2));
           const int zc = (x.l * P.B + x.b) * P.Hkv + x.h;
           for (int c = 0; c < SM::CH; ++c)
@@ -357,7 +343,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       int stage = 0;
       uint32_t phase = 0, bphase = 0, sphase = 0;   // bphase: one phase bit per accumulator
       long long prev = -1;
-      uint32_t idesc = idesc_bf16_f32(128, 128);
+      uint32_t idesc = 0;
       for (int sr = s_begin; sr < s_end; ++sr) {
         const int u = sr * S.ntiles + my_tile;
         const Unit x = decode(P, S, u);
@@ -367,7 +353,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           if (!mbar_wait(&sfull, sphase, abort_)) break;
           sphase ^= 1u;
           fence_after();
-          if (PASS == 2) idesc = idesc_bf16_f32(128, mass_block(P, S, x.tile).rows);
+          idesc = idesc_bf16_f32(128, mass_block(P, S, x.tile).rows);
           prev = key;
         }
         bool ok = true;
@@ -385,16 +371,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           for (int ks = 0; ks < D / 16; ++ks) {
             const int c = ks / 4, w = ks % 4;
             const uint64_t kd = sdesc_k_sw128(ks_base + c * BK * 128 + w * 32);
-            if (PASS == 1) {
-#pragma unroll
-              for (int m = 0; m < 2; ++m) {
-                const uint64_t pd = sdesc_k_sw128(st_base + c * SROWS * 128 + m * 128 * 128 + w * 32);
-                mma_bf16(dcol + m * 128, pd, kd, idesc, ks > 0 ? 1u : 0u);
-              }
-            } else {
-              const uint64_t pd = sdesc_k_sw128(st_base + c * SROWS * 128 + w * 32);
-              mma_bf16(dcol, kd, pd, idesc, ks > 0 ? 1u : 0u);
-            }
+            const uint64_t pd = sdesc_k_sw128(st_base + c * SROWS * 128 + w * 32);
+            mma_bf16(dcol, kd, pd, idesc, ks > 0 ? 1u : 0u);
           }
           mma_commit(&empty[stage]);
           mma_commit(&tfull[buf]);
@@ -406,18 +384,15 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    // Softmax pass: all four warpgroups drain every tile (warpgroup g takes
-    // M tile g & 1 and the 64-key half g >> 1), so while the CTA works on one
-    // accumulator the MMAs fill the other. Mass pass: warpgroups 0,1 drain
-    // accumulator 0 and 2,3 accumulator 1 (every other key tile), the two
-    // warpgroups of a pair splitting the groups of the stationary block.
-    // Either way every accumulator has a fixed set of consumers that waits
-    // for each of its phases in turn.
+    // Warpgroups 0,1 drain accumulator 0 and 2,3 accumulator 1 (every other
+    // key tile), the two warpgroups of a pair splitting the groups of the
+    // stationary block; each accumulator has one fixed pair of consumers
+    // that waits for each of its phases in turn.
     const int ew = warp - EPI_WARP0;      // 0..15
     const int wg = ew / 4;                // warpgroup 0..3
-    const int par = wg >> 1, sub = wg & 1;  // par: accumulator (mass) / key half (softmax)
+    const int par = wg >> 1, sub = wg & 1;  // accumulator / half of the block's groups
     const int q = warp % 4;               // TMEM lane quarter this warp may access
-    const int lrow = q * 32 + lane;       // accumulator lane: proxy row (1) / key (2)
+    const int lrow = q * 32 + lane;       // accumulator lane: a key of the tile
     const float alpha = P.alpha;
     uint32_t bphase = 0;                  // one phase bit per accumulator
     long long prev_blk = -1;
@@ -426,98 +401,281 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       const Unit x = decode(P, S, u);
       const ReqInfo R = P.req[x.b];
       const long long key = block_key(P, S, x);
-      // softmax pass: (reference max, sum of exp2(x - max)) of this thread's
-      // row over its tiles of this split; restarted per split so that the
-      // split's partial does not depend on what the CTA ran before
-      float m_run = -INFINITY, z_run = 0.f;
-      bool first = true;
-      Block blk{};
+      const Block blk = mass_block(P, S, x.tile);
       const float* cv = cs_all + ew * SROWS;   // this warp's copy of the block's negated normalisers
-      if (PASS == 2) {
-        blk = mass_block(P, S, x.tile);
-        if (key != prev_blk) {
-          const float* src = bf.cvals + (((size_t)x.l * P.B + x.b) * P.Hkv + x.h) * P.Prows_pad + blk.row0;
-          __syncwarp();
-          for (int i = lane; i < blk.rows; i += 32) cs_all[ew * SROWS + i] = -src[i];
-          __syncwarp();
-          prev_blk = key;
-        }
+      if (key != prev_blk) {
+        const float* src = bf.cvals + (((size_t)x.l * P.B + x.b) * P.Hkv + x.h) * P.Prows_pad + blk.row0;
+        __syncwarp();
+        for (int i = lane; i < blk.rows; i += 32) cs_all[ew * SROWS + i] = -src[i];
+        __syncwarp();
+        prev_blk = key;
       }
       bool ok = true;
       for (int kt = x.t0, j = 0; kt < x.t1; kt += BK, ++j) {
         const int buf = j & 1;
-        if (PASS == 2 && buf != par) continue;
+        if (buf != par) continue;
         const uint32_t ph = (bphase >> buf) & 1u;
         bphase ^= 1u << buf;
         if (!mbar_wait(&tfull[buf], ph, abort_)) { ok = false; break; }
         fence_after();
         const uint32_t tacc = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * ACC_STRIDE);
-        if (PASS == 1) {
-          const int c_lo = par * (BK / 2);           // this warpgroup's key half
-          const int nvalid = min(BK, x.t1 - kt) - c_lo;
-          const uint32_t tcol = tacc + (uint32_t)(sub * 128 + c_lo);
-          if (nvalid >= BK / 2) {        // every tile but the last of a short split
-#pragma unroll 1
-            for (int c0 = 0; c0 < BK / 2; c0 += 32) {
-              float v[32];
-              tmem_ld32(tcol + c0, v);
-              tmem_wait_ld();
-              if (first) {
-                softmax_first(v, alpha, m_run, z_run);
-                first = false;
-              } else {
-                softmax_chunk(v, alpha, m_run, z_run);
-              }
-            }
-          } else {
-#pragma unroll 1
-            for (int c0 = 0; c0 < BK / 2; c0 += 32) {
-              float v[32];
-              tmem_ld32(tcol + c0, v);
-              tmem_wait_ld();
-              mask_tail(v, c0, nvalid);
-              if (first) {
-                softmax_first(v, alpha, m_run, z_run);
-                first = false;
-              } else {
-                softmax_chunk(v, alpha, m_run, z_run);
-              }
-            }
-          }
-        } else {
-          const int t = kt + lrow;
-          const bool valid = t < x.t1;
-          const size_t col = (size_t)R.tok_off + t;
-          const int ng0 = (blk.ng + 1) / 2;
-          const int gb = sub == 0 ? 0 : ng0, ge = sub == 0 ? ng0 : blk.ng;
-          for (int gi = gb; gi < ge; ++gi) {
-            const float sm = group_sum(tacc + (uint32_t)(gi * P.RG), cv + gi * P.RG, P.RG, alpha);
-            if (valid)
-              bf.gmass[(((size_t)x.l * P.Hkv + x.h) * P.G + blk.g0 + gi) * P.total_T + col] = sm;
-          }
-          const bool my_anchor = blk.anchor && (blk.ng == 0 ? sub == 0 : sub == 1);
-          if (my_anchor) {
-            const int a0 = blk.ng * P.RG;
-            const float sm = group_sum(tacc + (uint32_t)a0, cv + a0, P.anchor_rows, alpha);
-            if (valid)
-              bf.anchor[((size_t)x.l * P.Hkv + x.h) * P.total_T + col] = sm / (float)P.r;
-          }
+        const int t = kt + lrow;
+        const bool valid = t < x.t1;
+        const size_t col = (size_t)R.tok_off + t;
+        const int ng0 = (blk.ng + 1) / 2;
+        const int gb = sub == 0 ? 0 : ng0, ge = sub == 0 ? ng0 : blk.ng;
+        for (int gi = gb; gi < ge; ++gi) {
+          const float sm = group_sum(tacc + (uint32_t)(gi * P.RG), cv + gi * P.RG, P.RG, alpha);
+          if (valid)
+            bf.gmass[(((size_t)x.l * P.Hkv + x.h) * P.G + blk.g0 + gi) * P.total_T + col] = sm;
+        }
+        const bool my_anchor = blk.anchor && (blk.ng == 0 ? sub == 0 : sub == 1);
+        if (my_anchor) {
+          const int a0 = blk.ng * P.RG;
+          const float sm = group_sum(tacc + (uint32_t)a0, cv + a0, P.anchor_rows, alpha);
+          if (valid)
+            bf.anchor[((size_t)x.l * P.Hkv + x.h) * P.total_T + col] = sm / (float)P.r;
         }
         fence_before();
         mbar_arrive(&tempty[buf]);
       }
       if (!ok) break;
-      if (PASS == 1) {
-        const int prow = x.tile * SROWS + sub * 128 + lrow;
-        bf.part[((((size_t)x.l * P.Hkv + x.h) * P.total_splits + R.split_off + x.split) * 2 + par) *
-                    P.Prows_pad + prow] = make_float2(m_run, z_run);
-      }
     }
   }
 
   fence_before();
   __syncthreads();
   if (warp == 1) tmem_dealloc(tmem, TMEM_COLS);
+  if (threadIdx.x == 0 && abort_flag) set_status(bf.status, kStatusTimeout);
+}
+
+// ---------------------------------------------------------------- softmax pass on CTA pairs
+// Each cluster of two CTAs (a pair) owns one 256-row stationary block: the
+// leader (rank 0) holds rows 0-127, the peer rows 128-255. K tiles have 256
+// keys; each CTA stages 128 of them (leader keys 0-127, peer 128-255). The
+// leader issues M = 256 x N = 256 pair MMAs, so per 16-deep K step each SM
+// reads 4 KB of its proxy rows and 4 KB of its keys from shared memory (half
+// of what a one-SM MMA pair of the same work reads); TMA completions of both
+// CTAs land on the leader's barriers, and its commits arrive on both CTAs'.
+// Each CTA's accumulator holds its 128 rows x 256 keys: warpgroup g drains
+// keys 64g .. 64g+63 of every tile, keeping one (max, sum) partial per row,
+// warpgroup and split (kUmmaPartSlots = 4 slots, merged in a fixed order).
+// Every epilogue warp of both CTAs releases the accumulator on the leader's
+// barrier once its tensor-memory reads have completed (tcgen05.wait::ld),
+// with a relaxed arrival.
+constexpr int PBK = 256;          // keys per K tile of the pair softmax pass
+constexpr int PROWS = 128;        // stationary rows per CTA of a pair
+constexpr int PNSTAGE = 6;        // K ring depth (each stage: 128 keys)
+
+template <int D>
+struct PairSmem {
+  static constexpr int CH = D / 64;
+  static constexpr int STAT_BYTES = CH * PROWS * 128;
+  static constexpr int STAGE_BYTES = CH * (PBK / 2) * 128;
+  static constexpr int RING_BYTES = PNSTAGE * STAGE_BYTES;
+  static constexpr int DYN_BYTES = 1024 + STAT_BYTES + RING_BYTES;
+};
+
+template <int D>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
+    softmax_pair_kernel(const __grid_constant__ CUtensorMap kmap,
+                        const __grid_constant__ CUtensorMap pmap, const __grid_constant__ Problem P,
+                        const __grid_constant__ Sched S, Buffers bf) {
+  using SM = PairSmem<D>;
+  extern __shared__ unsigned char smraw[];
+  unsigned char* sm =
+      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
+  unsigned char* stat = sm;
+  unsigned char* ring = sm + SM::STAT_BYTES;
+  // full / sfull / tempty count on the leader's copies; empty / sempty /
+  // tfull receive the leader's multicast commits in both CTAs
+  __shared__ uint64_t full[PNSTAGE], empty[PNSTAGE], sfull, sempty, tfull[2], tempty[2];
+  __shared__ uint32_t tbase;
+  __shared__ int abort_flag;
+  volatile int* abort_ = &abort_flag;
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const uint32_t rank = cluster_rank();
+  // team schedule as in the one-SM kernel, counted in pairs
+  const int pair = blockIdx.x >> 1;
+  const int nteams = (gridDim.x >> 1) / S.ntiles;
+  const int team = pair / S.ntiles, my_tile = pair % S.ntiles;
+  const int nsplit_rows = S.units / S.ntiles;
+  const int s_begin = (int)((long long)team * nsplit_rows / nteams);
+  const int s_end = (int)((long long)(team + 1) * nsplit_rows / nteams);
+
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    for (int s = 0; s < PNSTAGE; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(&sfull, 1);
+    mbar_init(&sempty, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&tfull[i], 1);
+      mbar_init(&tempty[i], 2 * (NEPI / 32));   // every epilogue warp of both CTAs
+    }
+    fence_barrier_init();
+    prefetch_tmap(&kmap);
+    prefetch_tmap(&pmap);
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(&tbase, TMEM_COLS);
+    tmem_relinquish_pair();
+  }
+  fence_before();
+  __syncthreads();
+  cluster_sync();   // both CTAs' barriers exist before any remote arrival
+  fence_after();
+  const uint32_t tmem = tbase;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer (both CTAs)
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0, sphase = 0;
+      long long prev = -1;
+      for (int sr = s_begin; sr < s_end; ++sr) {
+        const Unit x = decode(P, S, sr * S.ntiles + my_tile);
+        const long long key = block_key(P, S, x);
+        if (key != prev) {
+          if (!mbar_wait(&sempty, sphase ^ 1u, abort_)) break;
+          if (rank == 0) mbar_expect_tx(&sfull, (uint32_t)(2 * PROWS * D * 2));
+          const uint32_t bar = mapa(smem_u32(&sfull), 0);
+          const int zc = (x.l * P.B + x.b) * P.Hkv + x.h;
+          const int row0 = x.tile * SROWS + (int)rank * PROWS;
+          for (int c = 0; c < SM::CH; ++c)
+            for (int r = 0; r < PROWS; r += 16)
+              tma_load_3d_pair(stat + c * PROWS * 128 + r * 128, &pmap, bar, c * 64, row0 + r, zc);
+          sphase ^= 1u;
+          prev = key;
+        }
+        const int kbase = P.req[x.b].tok_off + (int)rank * (PBK / 2);
+        bool ok = true;
+        for (int kt = x.t0; kt < x.t1; kt += PBK) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_)) { ok = false; break; }
+          if (rank == 0) mbar_expect_tx(&full[stage], (uint32_t)(2 * SM::STAGE_BYTES));
+          const uint32_t bar = mapa(smem_u32(&full[stage]), 0);
+          for (int c = 0; c < SM::CH; ++c)
+            tma_load_3d_pair(ring + stage * SM::STAGE_BYTES + c * (PBK / 2) * 128, &kmap, bar,
+                             x.h * D + c * 64, kbase + kt, x.l);
+          if (++stage == PNSTAGE) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer (leader)
+    if (lane == 0 && rank == 0) {
+      int stage = 0;
+      uint32_t phase = 0, bphase = 0, sphase = 0;
+      long long prev = -1;
+      const uint32_t idesc = idesc_bf16_f32(2 * PROWS, PBK);
+      for (int sr = s_begin; sr < s_end; ++sr) {
+        const Unit x = decode(P, S, sr * S.ntiles + my_tile);
+        const long long key = block_key(P, S, x);
+        if (key != prev) {
+          if (prev != -1) mma_commit_pair(&sempty, 0x3);   // old block free once its MMAs finish
+          if (!mbar_wait(&sfull, sphase, abort_)) break;
+          sphase ^= 1u;
+          fence_after();
+          prev = key;
+        }
+        bool ok = true;
+        for (int kt = x.t0, j = 0; kt < x.t1; kt += PBK, ++j) {
+          const int buf = j & 1;
+          if (!mbar_wait(&full[stage], phase, abort_) ||
+              !mbar_wait(&tempty[buf], ((bphase >> buf) & 1u) ^ 1u, abort_)) { ok = false; break; }
+          fence_after();
+          const uint32_t ks_base = smem_u32(ring + stage * SM::STAGE_BYTES);
+          const uint32_t st_base = smem_u32(stat);
+          const uint32_t dcol = tmem + (uint32_t)(buf * PBK);
+#pragma unroll
+          for (int ks = 0; ks < D / 16; ++ks) {
+            const int c = ks / 4, w = ks % 4;
+            mma_bf16_pair(dcol, sdesc_k_sw128(st_base + c * PROWS * 128 + w * 32),
+                          sdesc_k_sw128(ks_base + c * (PBK / 2) * 128 + w * 32), idesc,
+                          ks > 0 ? 1u : 0u);
+          }
+          mma_commit_pair(&empty[stage], 0x3);
+          mma_commit_pair(&tfull[buf], 0x3);
+          if (++stage == PNSTAGE) { stage = 0; phase ^= 1u; }
+          bphase ^= 1u << buf;
+        }
+        if (!ok) break;
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue (both CTAs)
+    const int ew = warp - EPI_WARP0;
+    const int wg = ew / 4;                  // warpgroup: keys 64 wg .. of each tile
+    const int q = warp % 4;                 // TMEM lane quarter this warp may access
+    const int lrow = q * 32 + lane;         // accumulator lane: this CTA's proxy row
+    const float alpha = P.alpha;
+    const int c_lo = wg * (PBK / 4);
+    const uint32_t tempty_lead[2] = {mapa(smem_u32(&tempty[0]), 0), mapa(smem_u32(&tempty[1]), 0)};
+    uint32_t bphase = 0;
+    for (int sr = s_begin; sr < s_end; ++sr) {
+      const Unit x = decode(P, S, sr * S.ntiles + my_tile);
+      const ReqInfo R = P.req[x.b];
+      // (reference max, sum of exp2(x - max)) of this thread's row over its
+      // quarter of every tile of the split, restarted per split
+      float m_run = -INFINITY, z_run = 0.f;
+      bool first = true;
+      bool ok = true;
+      for (int kt = x.t0, j = 0; kt < x.t1; kt += PBK, ++j) {
+        const int buf = j & 1;
+        const uint32_t ph = (bphase >> buf) & 1u;
+        bphase ^= 1u << buf;
+        if (!mbar_wait(&tfull[buf], ph, abort_)) { ok = false; break; }
+        fence_after();
+        const uint32_t tcol =
+            tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * PBK + c_lo);
+        const int nvalid = min(PBK, x.t1 - kt) - c_lo;
+        if (nvalid >= PBK / 4) {         // every tile but the last of a short split
+#pragma unroll 1
+          for (int c0 = 0; c0 < PBK / 4; c0 += 32) {
+            float v[32];
+            tmem_ld32(tcol + c0, v);
+            tmem_wait_ld();
+            if (first) {
+              softmax_first(v, alpha, m_run, z_run);
+              first = false;
+            } else {
+              softmax_chunk(v, alpha, m_run, z_run);
+            }
+          }
+        } else {
+#pragma unroll 1
+          for (int c0 = 0; c0 < PBK / 4; c0 += 32) {
+            float v[32];
+            tmem_ld32(tcol + c0, v);
+            tmem_wait_ld();
+            mask_tail(v, c0, nvalid);
+            if (first) {
+              softmax_first(v, alpha, m_run, z_run);
+              first = false;
+            } else {
+              softmax_chunk(v, alpha, m_run, z_run);
+            }
+          }
+        }
+        fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster_relaxed(tempty_lead[buf]);
+      }
+      if (!ok) break;
+      const int prow = x.tile * SROWS + (int)rank * PROWS + lrow;
+      bf.part[((((size_t)x.l * P.Hkv + x.h) * P.total_splits + R.split_off + x.split) * kUmmaPartSlots +
+               wg) * P.Prows_pad + prow] = make_float2(m_run, z_run);
+    }
+  }
+
+  fence_before();
+  __syncthreads();
+  cluster_sync();   // no CTA leaves while the other may still reach its memory
+  if (warp == 1) tmem_dealloc_pair(tmem, TMEM_COLS);
   if (threadIdx.x == 0 && abort_flag) set_status(bf.status, kStatusTimeout);
 }
 
@@ -593,9 +751,9 @@ cudaError_t launch_d(const Problem& P, const Buffers& bf, cudaStream_t st, const
   const int nsm = sm_count();
   if (nsm <= 0) return cudaErrorInvalidDevice;
   cudaError_t e;
-  if ((e = cudaFuncSetAttribute(score_umma_kernel<1, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                SM::DYN_BYTES)) != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(score_umma_kernel<2, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  if ((e = cudaFuncSetAttribute(softmax_pair_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                PairSmem<D>::DYN_BYTES)) != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(mass_umma_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 SM::DYN_BYTES)) != cudaSuccess) return e;
   const Sched s1 = make_sched(P, 1), s2 = make_sched(P, 2);
   // whole teams of ntiles CTAs (one per stationary block), at most one CTA
@@ -607,15 +765,18 @@ cudaError_t launch_d(const Problem& P, const Buffers& bf, cudaStream_t st, const
   };
   if (ev && (e = cudaEventRecord(ev[1], st)) != cudaSuccess) return e;
   if (s1.units) {
-    score_umma_kernel<1, D><<<grid_of(s1), NTHREADS, SM::DYN_BYTES, st>>>(kmap, pmap, P,
-                                                                                      s1, bf);
+    // pairs of CTAs (clusters of two), whole teams of ntiles pairs
+    const int rows = s1.units / s1.ntiles;
+    const int nteams = std::max(1, std::min(nsm / (2 * s1.ntiles), rows));
+    softmax_pair_kernel<D><<<2 * nteams * s1.ntiles, NTHREADS, PairSmem<D>::DYN_BYTES, st>>>(
+        kmap, pmap, P, s1, bf);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   if (ev && (e = cudaEventRecord(ev[2], st)) != cudaSuccess) return e;
   if ((e = launch_merge(P, bf, st)) != cudaSuccess) return e;
   if (ev && (e = cudaEventRecord(ev[3], st)) != cudaSuccess) return e;
   if (s2.units) {
-    score_umma_kernel<2, D><<<grid_of(s2), NTHREADS, SM::DYN_BYTES, st>>>(kmap, pmap, P,
+    mass_umma_kernel<D><<<grid_of(s2), NTHREADS, SM::DYN_BYTES, st>>>(kmap, pmap, P,
                                                                                       s2, bf);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
