@@ -361,23 +361,47 @@ def run_gpu(args, wl):
     ok_h = torch.empty(out_k.shape, dtype=out_k.dtype, pin_memory=True)
     ov_h = torch.empty_like(ok_h, pin_memory=True)
     e_steps = max(1, args.steps)
+    # Every step copies its inputs from pinned host memory and reads its
+    # results back. The inputs are double-buffered on the device, so the
+    # copies of step k+1 (on a copy stream) overlap the selection of step k;
+    # a buffer is refilled only after the selection that read it.
+    Kb, Vb, Qb = [K, torch.empty_like(K)], [V, torch.empty_like(V)], [Q, torch.empty_like(Q)]
+    cstream = torch.cuda.Stream(dev)
+    ready = [torch.cuda.Event() for _ in range(2)]
+    free = [torch.cuda.Event() for _ in range(2)]
 
-    def e2e_step():
-        K.copy_(K_pin, non_blocking=True)
-        V.copy_(V_pin, non_blocking=True)
-        Q.copy_(Q_pin, non_blocking=True)
-        step()
+    def copy_in(i):
+        cstream.wait_event(free[i])
+        with torch.cuda.stream(cstream):
+            Kb[i].copy_(K_pin, non_blocking=True)
+            Vb[i].copy_(V_pin, non_blocking=True)
+            Qb[i].copy_(Q_pin, non_blocking=True)
+        ready[i].record(cstream)
+
+    def select_out(i):
+        stream.wait_event(ready[i])
+        M.check(M.mmshift_select(shape, Kb[i], Vb[i], Qb[i], None, params, out_idx, out_k, out_v,
+                                 None, ws, ws_bytes, stream), "mmshift_select")
+        free[i].record(stream)
         idx_h.copy_(out_idx, non_blocking=True)
         ok_h.copy_(out_k, non_blocking=True)
         ov_h.copy_(out_v, non_blocking=True)
 
-    e2e_step()                    # untimed warm-up of the pinned host buffers
+    def e2e(nsteps):
+        for ev in free:
+            ev.record(stream)
+        copy_in(0)
+        for k in range(nsteps):
+            if k + 1 < nsteps:
+                copy_in((k + 1) % 2)
+            select_out(k % 2)
+
+    e2e(2)                        # untimed warm-up of the pinned host buffers and streams
     torch.cuda.synchronize()
     ranks.barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    for _ in range(e_steps):
-        e2e_step()
+    e2e(e_steps)
     e1.record(stream)
     torch.cuda.synchronize()
     e_ms = ranks.max(e0.elapsed_time(e1) / e_steps, dev)
@@ -439,6 +463,8 @@ def run_gpu(args, wl):
         "roofline": roof,
         "cpu_baseline": cpu,
         "e2e": {"value": job_value(T * L, world, e_ms), "unit": UNIT, "ms_per_step": e_ms,
+                "pipeline": "inputs double-buffered on the device: the host-to-device copies "
+                            "of step k+1 overlap the selection of step k",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "clocks": clk,
         "gpu_launches": launches,
