@@ -115,6 +115,27 @@ def test_multi_layer_call_matches_single_layer_calls(lens):
             np.testing.assert_array_equal(multi[key][l], single[key][0], err_msg=key)
 
 
+# head_dim 64 in bf16 takes the tensor-core path too (softmax pass on CTA
+# pairs, mass pass with a separate anchor block and four groups per block)
+D64 = S.WORKLOADS["qwen7b-1layer"].replace(
+    name="d64-bf16", n_q_heads=8, n_kv_heads=2, head_dim=64, seq_lens=(3000, 1500),
+    n_visual=(2900, 1400), window=16, budgets=(256, 2000), n_centres=64, n_outlier=2)
+
+
+@pytest.mark.parametrize("kw", [dict(n_proxies=64, n_groups=4, score_mode=O.SCORE_VOTE),
+                                dict(n_proxies=64, n_groups=4, score_mode=O.SCORE_MASS),
+                                dict(n_proxies=512, n_groups=32)])
+def test_select_head_dim_64_tensor_cores(kw):
+    wl = D64
+    li = S.make_layer(wl, 0)
+    h = PT.hyper(**kw)
+    prox = S.make_proxies(wl, h["n_proxies"], 0)
+    gpu = PT.gpu_select(wl, [li], h, proxies=prox[None])
+    assert gpu["score_path"] == 1
+    refs = PT.oracle_layer(wl, li, h, 0, proxies=prox)
+    _check_all(wl, gpu, refs, h, what=f"d64 {kw}")
+
+
 # ---------------------------------------------------------------------------
 # end to end with the sampled proxies
 # ---------------------------------------------------------------------------
