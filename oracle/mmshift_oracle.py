@@ -31,7 +31,8 @@ F32 = "f32"
 
 __all__ = [
     "DEFAULTS", "SCORE_VOTE", "SCORE_MASS", "BF16", "F32", "philox4x64_10", "uniforms_from_bits",
-    "proxy_normals", "window_stats", "rope_rotate", "round_to", "build_proxies",
+    "proxy_normals", "window_stats", "prefill_stats", "rope_rotate", "round_to",
+    "build_proxies", "build_proxies_from_stats",
     "softmax_rows", "group_masses", "anchor_attention", "cover_sets", "votes",
     "scores", "select_topk", "gather", "select_request", "select",
 ]
@@ -145,6 +146,23 @@ def window_stats(qwin: np.ndarray):
     return mu, np.sqrt(var)
 
 
+def prefill_stats(qfull: np.ndarray):
+    """Statistics over the whole prefill (§3.2.1: mu_pre and sigma_pre are taken
+    across all prompt tokens).
+
+    Reading: in query space, per (query head, dimension) over all T prompt
+    queries of the request, with the unbiased (T - 1) estimator (0 for T = 1).
+    qfull: [T, Hq, d] -> (mu, sigma), each [Hq, d] float64.
+    """
+    q = np.asarray(qfull, dtype=np.float64)
+    t = q.shape[0]
+    mu = q.sum(axis=0) / t
+    if t < 2:
+        return mu, np.zeros_like(mu)
+    var = ((q - mu) ** 2).sum(axis=0) / (t - 1)
+    return mu, np.sqrt(var)
+
+
 def rope_rotate(x: np.ndarray, pos: float, theta: float) -> np.ndarray:
     """Rotary embedding at position ``pos`` (rotate-half pairing).
 
@@ -184,6 +202,17 @@ def build_proxies(qwin: np.ndarray, z: np.ndarray, gamma: float, t_len: int,
     qwin: [W, Hq, d]; z: [Hq, N_p, d] -> [Hq, N_p, d] float64 (dtype-exact).
     """
     mu, sigma = window_stats(qwin)
+    return build_proxies_from_stats(mu, sigma, z, gamma, t_len, dtype, rope_theta, rope_pos_offset)
+
+
+def build_proxies_from_stats(mu: np.ndarray, sigma: np.ndarray, z: np.ndarray, gamma: float,
+                             t_len: int, dtype: str, rope_theta: float = 0.0,
+                             rope_pos_offset: int = 0):
+    """The same expansion from given statistics (e.g. prefill_stats):
+    q~[hq, i, j] = mu[hq, j] + gamma * sigma[hq, j] * z[hq, i, j], then the
+    optional RoPE rotation and rounding of build_proxies.
+    mu, sigma: [Hq, d]; z: [Hq, N_p, d] -> [Hq, N_p, d] float64 (dtype-exact).
+    """
     q = mu[:, None, :] + gamma * sigma[:, None, :] * z
     if rope_theta > 0.0:
         q = rope_rotate(q, float(t_len + rope_pos_offset), rope_theta)
@@ -315,13 +344,16 @@ def gather(keys: np.ndarray, values: np.ndarray, idx: np.ndarray):
 def select_request(keys, values, qwin, budget: int, *, n_proxies=512, n_groups=32,
                    gamma=10.0, tau=0.95, lam=1.0, seed=0, layer_id=0, b=0,
                    score_mode=SCORE_VOTE, softmax_scale=0.0, rope_theta=0.0,
-                   rope_pos_offset=0, dtype=BF16, proxies=None) -> Dict[str, np.ndarray]:
+                   rope_pos_offset=0, dtype=BF16, proxies=None,
+                   qfull=None) -> Dict[str, np.ndarray]:
     """Algorithm 1 for one request of one layer.
 
     keys/values: [T, Hkv, d]; qwin: [W, Hq, d] (its last row is the last real
     prefill query). ``proxies`` ([Hq, N_p, d]) replaces the sampled proxies
-    when given. Returns proxies, group masses, anchor, mass, scores, indices
-    ([C', Hkv], ascending per head) and the gathered cache.
+    when given. ``qfull`` ([T, Hq, d], all prompt queries), when given, is the
+    source of the proxies' statistics (prefill_stats) instead of the window.
+    Returns proxies, group masses, anchor, mass, scores, indices ([C', Hkv],
+    ascending per head) and the gathered cache.
     """
     keys = np.asarray(keys, dtype=np.float64)
     values = np.asarray(values, dtype=np.float64)
@@ -331,7 +363,12 @@ def select_request(keys, values, qwin, budget: int, *, n_proxies=512, n_groups=3
     scale = softmax_scale if softmax_scale > 0.0 else 1.0 / math.sqrt(d)
     if proxies is None:
         z = proxy_normals(seed, layer_id, b, hq, n_proxies, d)
-        proxies = build_proxies(qwin, z, gamma, t_len, dtype, rope_theta, rope_pos_offset)
+        if qfull is None:
+            proxies = build_proxies(qwin, z, gamma, t_len, dtype, rope_theta, rope_pos_offset)
+        else:
+            mu, sigma = prefill_stats(qfull)
+            proxies = build_proxies_from_stats(mu, sigma, z, gamma, t_len, dtype, rope_theta,
+                                               rope_pos_offset)
     else:
         proxies = np.asarray(proxies, dtype=np.float64)
     abar = group_masses(proxies, keys, n_groups, scale)            # [Hkv, G, T]

@@ -17,6 +17,16 @@ def _window_stats_ddof0(qwin):
     return mu, q.std(axis=0)
 
 
+def _prefill_stats_ddof0(qfull):
+    q = np.asarray(qfull, dtype=np.float64)
+    return q.mean(axis=0), q.std(axis=0)
+
+
+def _proxies_from_stats_sigma_squared(mu, sigma, z, gamma, t_len, dtype, rope_theta=0.0,
+                                      rope_pos_offset=0):
+    return O.round_to(mu[:, None, :] + gamma * (sigma ** 2)[:, None, :] * z, dtype)
+
+
 def _build_proxies_no_gamma(qwin, z, gamma, t_len, dtype, rope_theta=0.0, rope_pos_offset=0):
     mu, sigma = O.window_stats(qwin)
     return O.round_to(mu[:, None, :] + sigma[:, None, :] * z, dtype)
@@ -118,6 +128,8 @@ def _philox_9_rounds(ctr, key):
 
 MUTANTS = {
     "std_ddof0": ("window_stats", _window_stats_ddof0),
+    "prefill_std_ddof0": ("prefill_stats", _prefill_stats_ddof0),
+    "proxies_variance_not_std": ("build_proxies_from_stats", _proxies_from_stats_sigma_squared),
     "no_gamma": ("build_proxies", _build_proxies_no_gamma),
     "gqa_modulo_mapping": ("group_masses", _group_masses_wrong_gqa),
     "no_softmax_scale": ("group_masses", _group_masses_no_scale),

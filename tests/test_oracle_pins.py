@@ -68,6 +68,34 @@ def pin_window_stats(orc=O):
             assert math.isclose(sigma[h, j], statistics.stdev(col), rel_tol=1e-12)
 
 
+def pin_prefill_stats(orc=O):
+    """§3.2.1 statistics across all prompt tokens: against a second
+    implementation (the statistics module), the closed form of an arithmetic
+    progression, the single-token case, and the window path as the special
+    case of a prompt that is its own window."""
+    rng = np.random.default_rng(21)
+    q = rng.normal(size=(37, 2, 4)) * 2.0 - 0.5
+    mu, sigma = orc.prefill_stats(q)
+    for h in range(2):
+        for j in range(4):
+            col = [float(v) for v in q[:, h, j]]
+            assert math.isclose(mu[h, j], statistics.fmean(col), rel_tol=1e-12, abs_tol=1e-12)
+            assert math.isclose(sigma[h, j], statistics.stdev(col), rel_tol=1e-12)
+    # x_t = a + c t, t < T: mean a + c (T - 1) / 2, unbiased variance c^2 T (T + 1) / 12
+    t_len, a, c = 1000, 0.25, -0.003
+    ap = (a + c * np.arange(t_len))[:, None, None] * np.ones((1, 1, 3))
+    mu, sigma = orc.prefill_stats(ap)
+    assert np.allclose(mu, a + c * (t_len - 1) / 2, rtol=1e-12, atol=1e-15)
+    assert np.allclose(sigma ** 2, c * c * t_len * (t_len + 1) / 12, rtol=1e-10)
+    mu, sigma = orc.prefill_stats(q[:1])
+    assert np.array_equal(mu, q[0]) and np.all(sigma == 0)
+    qwin = rng.normal(size=(16, 2, 8))
+    z = orc.proxy_normals(seed=5, layer_id=1, b=0, n_q_heads=2, n_proxies=32, head_dim=8)
+    w = orc.build_proxies(qwin, z, 3.0, 50, orc.BF16)
+    m, sg = orc.prefill_stats(qwin)
+    assert np.array_equal(w, orc.build_proxies_from_stats(m, sg, z, 3.0, 50, orc.BF16))
+
+
 def pin_sampler_closed_form(orc=O):
     """Appendix A.2: for q ~ N(mu, Sigma), E[exp(q.k/sqrt d)] =
     exp(mu.k/sqrt d + k^T Sigma k / (2d)). With Sigma = diag((gamma*sigma)^2)
@@ -288,7 +316,7 @@ def pin_topk_bruteforce(orc=O):
             assert cand == list(bests[0])
 
 
-ALL_PINS = [pin_philox_vs_numpy, pin_normals_distribution, pin_window_stats,
+ALL_PINS = [pin_philox_vs_numpy, pin_normals_distribution, pin_window_stats, pin_prefill_stats,
             pin_sampler_closed_form, pin_rope, pin_round_bf16, pin_mass_totals,
             pin_sigma_zero_single_query, pin_shift_and_permutation, pin_budget_ge_t,
             pin_lastattn, pin_uniform_keys, pin_cover_bruteforce, pin_topk_bruteforce]
