@@ -13,6 +13,11 @@ Metric: prompt tokens selected per second per layer (sum_b T_b * L / step
 time), whole job over all ranks; plus the fraction of the HBM roofline the
 step's algorithmic bytes (K read once + K/V gathered, read and written) reach.
 
+--stats prefill takes the proxies' statistics over every prompt query instead
+of the window's (Section 3.2.1): each step then also reads the L x T x Hq x d
+prompt queries once (mmshift_prefill_stats) and selects with
+mmshift_select_with_stats; the line adds that pass's HBM roofline.
+
 --impl reference times the CPU oracle on the host cores instead (a bounded
 sample of the same workload per step).
 
@@ -71,6 +76,33 @@ def gen_workload(wl, rank_seed: int, procs: int):
     else:
         parts = [_gen_one(j) for j in jobs]
     return tuple(np.stack([p[i] for p in parts]) for i in range(3))
+
+
+def prompt_queries_device(wl, K, Qwin, seed: int):
+    """All prompt queries [L, T*Hq*d] on the device for --stats prefill, with
+    the recipe of synth.make_prompt_queries (half the request's per-head key
+    mean plus unit normal noise, a N(0, 1) modality offset per (head,
+    dimension) on visual positions, the window queries as the last rows),
+    drawn by torch's seeded device generator: the 28 x 32K x 28 x 128 stack
+    is 6.6 GB, too large to draw on the host every run."""
+    import torch
+    L, T = wl.n_layers, wl.total_tokens
+    hq, hkv, d, w = wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.window
+    g = torch.Generator(device=K.device).manual_seed(seed)
+    out = torch.empty((L, T, hq, d), dtype=K.dtype, device=K.device)
+    cu = wl.cu_seqlens()
+    Kv = K.view(L, T, hkv, d)
+    Qv = Qwin.view(L, wl.batch, w, hq, d)
+    for l in range(L):
+        for b, (t_len, n_vis) in enumerate(zip(wl.seq_lens, wl.n_visual)):
+            lo, hi = int(cu[b]), int(cu[b + 1])
+            kmean = Kv[l, lo:hi].float().mean(dim=0).repeat_interleave(hq // hkv, dim=0)
+            q = torch.randn((t_len, hq, d), generator=g, device=K.device) + 0.5 * kmean
+            q[:n_vis] += torch.randn((hq, d), generator=g, device=K.device)
+            out[l, lo:hi] = q.to(K.dtype)
+            nw = min(w, t_len)
+            out[l, hi - nw:hi] = Qv[l, b, w - nw:]
+    return out.view(L, -1)
 
 
 def read_peaks():
@@ -322,10 +354,29 @@ def run_gpu(args, wl):
     out_v = torch.empty_like(out_k)
     stream = torch.cuda.current_stream(dev)
     nst = LB.MMSHIFT_N_STAGES + 1
+    prefill = args.stats == "prefill"
+    if prefill:
+        Qf = prompt_queries_device(wl, K, Q, seed=wl.seed + 7919 * (rank + 1))
+        st_bytes = M.mmshift_prefill_stats_workspace_size(shape)
+        st_ws = torch.zeros(st_bytes, dtype=torch.uint8, device=dev)
+        stats = torch.empty((L, wl.batch, 2, wl.n_q_heads * wl.head_dim), device=dev)
 
-    def step(dbg=None):
-        M.check(M.mmshift_select(shape, K, V, Q, None, params, out_idx, out_k, out_v, dbg, ws,
-                                 ws_bytes, stream), "mmshift_select")
+    def select(Kx, Vx, Qx, Qfx, dbg=None, sev=None):
+        if not prefill:
+            M.check(M.mmshift_select(shape, Kx, Vx, Qx, None, params, out_idx, out_k, out_v, dbg,
+                                     ws, ws_bytes, stream), "mmshift_select")
+            return
+        if sev:
+            sev[0].record(stream)
+        M.check(M.mmshift_prefill_stats(shape, Qfx, 0, stats, st_ws, st_bytes, stream),
+                "mmshift_prefill_stats")
+        if sev:
+            sev[1].record(stream)
+        M.check(M.mmshift_select_with_stats(shape, Kx, Vx, Qx, stats, params, out_idx, out_k, out_v,
+                                            dbg, ws, ws_bytes, stream), "mmshift_select_with_stats")
+
+    def step(dbg=None, sev=None):
+        select(K, V, Q, Qf if prefill else None, dbg, sev)
 
     for _ in range(args.warmup):
         step()
@@ -337,6 +388,8 @@ def run_gpu(args, wl):
         for ev in evs:
             ev.record(stream)
     dbgs = [M.make_debug(stage_events=ev) for ev in stage_ev]
+    stat_ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] if prefill else None
+               for _ in range(args.steps)]
     clocks = ClockSampler(torch.cuda.current_device())
     clocks.start()
     time.sleep(0.3)
@@ -345,7 +398,7 @@ def run_gpu(args, wl):
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     t_start.record(stream)
     for k in range(args.steps):
-        step(dbgs[k])
+        step(dbgs[k], stat_ev[k])
     t_end.record(stream)
     torch.cuda.synchronize()
     ranks.barrier()
@@ -355,6 +408,10 @@ def run_gpu(args, wl):
     stage_ms = {name: statistics.mean(ev[i].elapsed_time(ev[i + 1]) for ev in stage_ev)
                 for i, name in enumerate(LB.STAGES)}
     launches = dbgs[0].launches * args.steps
+    if prefill:
+        stage_ms = {"prefill_stats": statistics.mean(e[0].elapsed_time(e[1]) for e in stat_ev),
+                    **stage_ms}
+        launches += 2 * args.steps        # partial sums + merge
 
     # end to end through the same C ABI call: host buffers in, results out
     idx_h = torch.empty(out_idx.shape, dtype=out_idx.dtype, pin_memory=True)
@@ -366,6 +423,10 @@ def run_gpu(args, wl):
     # copies of step k+1 (on a copy stream) overlap the selection of step k;
     # a buffer is refilled only after the selection that read it.
     Kb, Vb, Qb = [K, torch.empty_like(K)], [V, torch.empty_like(V)], [Q, torch.empty_like(Q)]
+    if prefill:
+        Qf_pin = torch.empty(Qf.shape, dtype=Qf.dtype, pin_memory=True)
+        Qf_pin.copy_(Qf)
+        Qfb = [Qf, torch.empty_like(Qf)]
     cstream = torch.cuda.Stream(dev)
     ready = [torch.cuda.Event() for _ in range(2)]
     free = [torch.cuda.Event() for _ in range(2)]
@@ -376,12 +437,13 @@ def run_gpu(args, wl):
             Kb[i].copy_(K_pin, non_blocking=True)
             Vb[i].copy_(V_pin, non_blocking=True)
             Qb[i].copy_(Q_pin, non_blocking=True)
+            if prefill:
+                Qfb[i].copy_(Qf_pin, non_blocking=True)
         ready[i].record(cstream)
 
     def select_out(i):
         stream.wait_event(ready[i])
-        M.check(M.mmshift_select(shape, Kb[i], Vb[i], Qb[i], None, params, out_idx, out_k, out_v,
-                                 None, ws, ws_bytes, stream), "mmshift_select")
+        select(Kb[i], Vb[i], Qb[i], Qfb[i] if prefill else None)
         free[i].record(stream)
         idx_h.copy_(out_idx, non_blocking=True)
         ok_h.copy_(out_k, non_blocking=True)
@@ -406,9 +468,24 @@ def run_gpu(args, wl):
     torch.cuda.synchronize()
     e_ms = ranks.max(e0.elapsed_time(e1) / e_steps, dev)
     h2d = sum(t.numel() * t.element_size() for t in (K_pin, V_pin, Q_pin))
+    if prefill:
+        h2d += Qf_pin.numel() * Qf_pin.element_size()
     d2h = sum(t.numel() * t.element_size() for t in (idx_h, ok_h, ov_h))
 
     bytes_step, k_read, pass_flops = algorithmic(wl, hyper)
+    stats_roof = None
+    if prefill:
+        # algorithmic bytes of the statistics pass: every prompt query read
+        # once, the [L, B, 2, Hq*d] float32 statistics written
+        q_bytes = Qf.numel() * Qf.element_size()
+        s_bytes = q_bytes + stats.numel() * 4
+        bytes_step += q_bytes
+        st_ms = stage_ms["prefill_stats"]
+        ach = s_bytes / (st_ms * 1e-3) / 1e9
+        stats_roof = {"bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                      "frac": ach / peaks["hbm_gbs"], "traffic": None,
+                      "kernel": "stats_partial_kernel + stats_merge_kernel",
+                      "bytes_per_launch": s_bytes, "peak_kind": f"HBM copy ({peak_src})"}
     tokens_layer = T * L * world          # metric unit: tokens per second per layer
     value = job_value(T * L, world, ms)
     hbm_frac = bytes_step / (ms * 1e-3) / (peaks["hbm_gbs"] * 1e9)
@@ -455,12 +532,14 @@ def run_gpu(args, wl):
                    "window": wl.window, "budgets": list(wl.budgets), "proxies": args.proxies,
                    "n_proxies": hyper["n_proxies"], "n_groups": hyper["n_groups"],
                    "gamma": hyper["gamma"], "tau": hyper["tau"], "lambda": hyper["lam"],
+                   "stats": args.stats,
                    "l2": "inputs (K+V %.2f GB) larger than L2; no flush" % (2 * k_read / 1e9),
                    "parallelism": f"replicas x{world}"},
         "hbm_roofline_frac": hbm_frac,
         "hbm_bytes_per_step": bytes_step,
         "stage_ms": stage_ms,
         "roofline": roof,
+        **({"prefill_stats_roofline": stats_roof} if stats_roof else {}),
         "cpu_baseline": cpu,
         "e2e": {"value": job_value(T * L, world, e_ms), "unit": UNIT, "ms_per_step": e_ms,
                 "pipeline": "inputs double-buffered on the device: the host-to-device copies "
@@ -487,6 +566,9 @@ def main(argv=None):
                     help="use only the first N layers of the workload (profiling runs)")
     ap.add_argument("--proxies", choices=["paper", "few"], default="paper",
                     help="paper: N=512, G=32 (Section 4.1); few: N=W, G=W/16")
+    ap.add_argument("--stats", choices=["window", "prefill"], default="window",
+                    help="proxy statistics: over the W window queries, or over every prompt "
+                         "query (mmshift_prefill_stats + mmshift_select_with_stats)")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="CPU oracle sample budget for cpu_baseline (0 disables)")
     ap.add_argument("--ref-seconds", type=float, default=8.0,

@@ -152,6 +152,33 @@ mmshift_status mmshift_build_proxies(const mmshift_shape* s, const void* Qwin,
                                      const mmshift_params* p, void* proxies,
                                      mmshift_stream_t stream);
 
+/* Proxy statistics over the whole prefill (Section 3.2.1: the mean and the
+ * standard deviation of the prompt's features are taken across all prompt
+ * tokens; read in query space): for every layer l, request b, query head hq
+ * and dimension j, over the T_b prompt queries of the request,
+ *   stats[l][b][0][hq][j] = mean_t Qfull[l][cu_b + t][hq][j],
+ *   stats[l][b][1][hq][j] = their standard deviation, T_b - 1 denominator
+ *                           (0 for T_b = 1).
+ * Qfull: [L][total_T][Hq][d] in the shape's dtype, 16-byte aligned; layers
+ * `qfull_layer_stride` elements apart (0 = densely packed; a multiple of 8).
+ * stats: [L][batch][2][Hq][d] float32. workspace: at least
+ * mmshift_prefill_stats_workspace_size() bytes (per-chunk partial sums).
+ * Reads every byte of Qfull once; deterministic (fixed merge order). */
+mmshift_status mmshift_prefill_stats_workspace_size(const mmshift_shape* s, size_t* bytes);
+mmshift_status mmshift_prefill_stats(const mmshift_shape* s, const void* Qfull,
+                                     int64_t qfull_layer_stride, float* stats, void* workspace,
+                                     size_t workspace_bytes, mmshift_stream_t stream);
+
+/* Step 1 from given statistics (e.g. mmshift_prefill_stats) instead of the
+ * observation window's: q~ = mu + gamma * sigma * z with the same normals,
+ * RoPE and rounding as mmshift_build_proxies. stats: [L][batch][2][Hq][d]
+ * float32 (mean, std); proxies: [L, batch, Hq, N, d]. Pass the proxies to
+ * mmshift_select / mmshift_proxy_mass to select with them, or pass the
+ * statistics to mmshift_select_with_stats. */
+mmshift_status mmshift_build_proxies_from_stats(const mmshift_shape* s, const float* stats,
+                                                const mmshift_params* p, void* proxies,
+                                                mmshift_stream_t stream);
+
 /* Steps 2-4 (Section 3.2.2, Appendix B): softmax attention of every proxy over
  * all T_b keys of its KV head (h = hq / r), summed per proxy group over the r
  * query heads of that KV head; and the last-query anchor (mean over the r
@@ -201,6 +228,18 @@ mmshift_status mmshift_select(const mmshift_shape* s, const void* K, const void*
                               const mmshift_params* p, int32_t* out_idx, void* out_K,
                               void* out_V, const mmshift_debug* dbg, void* workspace,
                               size_t workspace_bytes, mmshift_stream_t stream);
+
+/* mmshift_select with the proxies' statistics given (Section 3.2.1: mean and
+ * std over the whole prefill, e.g. from mmshift_prefill_stats) instead of
+ * taken over the observation window; the sampled proxies use the same normals,
+ * RoPE and rounding. stats: [L][batch][2][Hq][d] float32 (mean, std), read
+ * only, must not be NULL. Qwin still supplies the anchor (its last row).
+ * Same outputs, workspace and errors as mmshift_select. */
+mmshift_status mmshift_select_with_stats(const mmshift_shape* s, const void* K, const void* V,
+                                         const void* Qwin, const float* stats,
+                                         const mmshift_params* p, int32_t* out_idx, void* out_K,
+                                         void* out_V, const mmshift_debug* dbg, void* workspace,
+                                         size_t workspace_bytes, mmshift_stream_t stream);
 
 /* Allocation-free variant of mmshift_scores_topk.
  *

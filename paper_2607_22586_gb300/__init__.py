@@ -10,4 +10,6 @@ from . import synth  # noqa: F401
 from ._lib import (MMShiftError, Params, Shape, Debug, check, default_params,  # noqa: F401
                    load_library, make_debug, make_shape, mmshift_build_proxies, mmshift_gather,
                    mmshift_output_rows, mmshift_poll_status, mmshift_proxy_mass,
-                   mmshift_scores_topk, mmshift_scores_topk_noalloc, mmshift_select, mmshift_topk, mmshift_workspace_size)
+                   mmshift_scores_topk, mmshift_scores_topk_noalloc, mmshift_select, mmshift_topk,
+                   mmshift_workspace_size, mmshift_prefill_stats, mmshift_prefill_stats_workspace_size,
+                   mmshift_build_proxies_from_stats, mmshift_select_with_stats)

@@ -32,6 +32,8 @@ EXPORTED = [
     "mmshift_build_proxies", "mmshift_proxy_mass", "mmshift_scores_topk", "mmshift_topk",
     "mmshift_gather", "mmshift_select", "mmshift_poll_status", "mmshift_status_string",
     "mmshift_last_cuda_error", "mmshift_scores_topk_noalloc",
+    "mmshift_prefill_stats_workspace_size", "mmshift_prefill_stats",
+    "mmshift_build_proxies_from_stats", "mmshift_select_with_stats",
 ]
 MMSHIFT_NOALLOC_SCRATCH_BYTES = 8 << 20
 
@@ -94,6 +96,12 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.mmshift_workspace_size.restype = st
     lib.mmshift_build_proxies.argtypes = [_SP, _VP, _PP, _VP, _VP]
     lib.mmshift_build_proxies.restype = st
+    lib.mmshift_prefill_stats_workspace_size.argtypes = [_SP, ctypes.POINTER(ctypes.c_size_t)]
+    lib.mmshift_prefill_stats_workspace_size.restype = st
+    lib.mmshift_prefill_stats.argtypes = [_SP, _VP, ctypes.c_int64, _VP, _VP, ctypes.c_size_t, _VP]
+    lib.mmshift_prefill_stats.restype = st
+    lib.mmshift_build_proxies_from_stats.argtypes = [_SP, _VP, _PP, _VP, _VP]
+    lib.mmshift_build_proxies_from_stats.restype = st
     lib.mmshift_proxy_mass.argtypes = [_SP, _VP, _VP, _VP, _PP, _VP, _VP, _VP, _VP, ctypes.c_size_t, _VP]
     lib.mmshift_proxy_mass.restype = st
     lib.mmshift_scores_topk.argtypes = [_SP, _PP, _VP, _VP, _VP, _VP, _VP, ctypes.c_size_t, _VP]
@@ -105,6 +113,9 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.mmshift_select.argtypes = [_SP, _VP, _VP, _VP, _VP, _PP, _VP, _VP, _VP,
                                    ctypes.POINTER(Debug), _VP, ctypes.c_size_t, _VP]
     lib.mmshift_select.restype = st
+    lib.mmshift_select_with_stats.argtypes = [_SP, _VP, _VP, _VP, _VP, _PP, _VP, _VP, _VP,
+                                              ctypes.POINTER(Debug), _VP, ctypes.c_size_t, _VP]
+    lib.mmshift_select_with_stats.restype = st
     lib.mmshift_scores_topk_noalloc.argtypes = [_SP, _PP, _VP, _VP, _VP, _VP, _VP]
     lib.mmshift_scores_topk_noalloc.restype = st
     lib.mmshift_poll_status.argtypes = [_VP, _VP]
@@ -182,6 +193,26 @@ def mmshift_build_proxies(shape, qwin, params, proxies, stream=None) -> int:
                                                 _ptr(proxies), _ptr(stream))
 
 
+def mmshift_prefill_stats_workspace_size(shape: Shape) -> int:
+    n = ctypes.c_size_t()
+    check(load_library().mmshift_prefill_stats_workspace_size(ctypes.byref(shape), ctypes.byref(n)),
+          "mmshift_prefill_stats_workspace_size")
+    return n.value
+
+
+def mmshift_prefill_stats(shape, qfull, qfull_layer_stride, stats, workspace, workspace_bytes,
+                          stream=None) -> int:
+    return load_library().mmshift_prefill_stats(ctypes.byref(shape), _ptr(qfull),
+                                                int(qfull_layer_stride), _ptr(stats),
+                                                _ptr(workspace), workspace_bytes, _ptr(stream))
+
+
+def mmshift_build_proxies_from_stats(shape, stats, params, proxies, stream=None) -> int:
+    return load_library().mmshift_build_proxies_from_stats(ctypes.byref(shape), _ptr(stats),
+                                                           ctypes.byref(params), _ptr(proxies),
+                                                           _ptr(stream))
+
+
 def mmshift_proxy_mass(shape, K, qwin, proxies, params, group_mass, anchor, mass, workspace,
                        workspace_bytes, stream=None) -> int:
     return load_library().mmshift_proxy_mass(
@@ -221,6 +252,15 @@ def mmshift_select(shape, K, V, qwin, proxies_in, params, out_idx, out_K, out_V,
     dbg = ctypes.byref(debug) if debug is not None else None
     return load_library().mmshift_select(
         ctypes.byref(shape), _ptr(K), _ptr(V), _ptr(qwin), _ptr(proxies_in), ctypes.byref(params),
+        _ptr(out_idx), _ptr(out_K), _ptr(out_V), dbg, _ptr(workspace), workspace_bytes, _ptr(stream))
+
+
+
+def mmshift_select_with_stats(shape, K, V, qwin, stats, params, out_idx, out_K, out_V, debug,
+                              workspace, workspace_bytes, stream=None) -> int:
+    dbg = ctypes.byref(debug) if debug is not None else None
+    return load_library().mmshift_select_with_stats(
+        ctypes.byref(shape), _ptr(K), _ptr(V), _ptr(qwin), _ptr(stats), ctypes.byref(params),
         _ptr(out_idx), _ptr(out_K), _ptr(out_V), dbg, _ptr(workspace), workspace_bytes, _ptr(stream))
 
 

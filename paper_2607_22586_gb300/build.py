@@ -19,7 +19,8 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libmmshift.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["api.cu", "proxy.cu", "score_simt.cu", "score_umma.cu", "select.cu", "noalloc.cu"]
+SOURCES = ["api.cu", "proxy.cu", "score_simt.cu", "score_umma.cu", "select.cu", "stats.cu",
+           "noalloc.cu"]
 
 
 def _nvcc() -> str:

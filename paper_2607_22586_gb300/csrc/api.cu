@@ -1,6 +1,7 @@
 // Host side of the C ABI declared in include/mmshift.h: argument validation,
 // problem description, workspace carve-up and kernel sequencing. Nothing here
 // allocates device memory or synchronises (except mmshift_poll_status).
+#include <algorithm>
 #include <cmath>
 #include <cstring>
 #include <string>
@@ -232,6 +233,70 @@ mmshift_status noalloc_prepare(const mmshift_shape* s, const mmshift_params* p, 
 mmshift_status noalloc_cuda_fail(cudaError_t e) { return cuda_fail(e); }
 }  // namespace mmshift
 
+// Whole-prefill statistics job of a shape (no hyper-parameters involved).
+static mmshift_status stats_job(const mmshift_shape* s, int64_t qfull_layer_stride, StatsJob* J) {
+  mmshift_status st = check_shape(s);
+  if (st != MMSHIFT_OK) return st;
+  std::memset(J, 0, sizeof(*J));
+  J->L = s->n_layers;
+  J->B = s->batch;
+  J->ncol = s->n_q_heads * s->head_dim;
+  const int64_t total = s->cu_seqlens[s->batch];
+  int maxc = 0;
+  for (int b = 0; b < s->batch; ++b) {
+    J->tok_off[b] = s->cu_seqlens[b];
+    J->t_len[b] = s->cu_seqlens[b + 1] - s->cu_seqlens[b];
+    maxc = std::max(maxc, (J->t_len[b] + kStatsChunk - 1) / kStatsChunk);
+  }
+  J->nchunk = maxc;
+  const int64_t dense = total * J->ncol;
+  J->ls = qfull_layer_stride ? qfull_layer_stride : dense;
+  if (J->L > 1 && J->ls < dense) return MMSHIFT_ERR_INVALID_ARG;
+  if (J->ls % 8) return MMSHIFT_ERR_INVALID_ARG;   // 16-byte rows for the vector loads
+  return MMSHIFT_OK;
+}
+
+// Steps 1-6 of Algorithm 1 for every layer; proxies from the window
+// statistics, from given statistics (stats_in) or given outright (proxies_in).
+static mmshift_status select_impl(const mmshift_shape* s, const void* K, const void* V,
+                                  const void* Qwin, const void* proxies_in, const float* stats_in,
+                                  const mmshift_params* p, int32_t* out_idx, void* out_K,
+                                  void* out_V, const mmshift_debug* dbg, void* workspace,
+                                  size_t workspace_bytes, mmshift_stream_t stream) {
+  Problem P;
+  mmshift_status st = prepare(s, p, &P);
+  if (st != MMSHIFT_OK) return st;
+  if (!p || !K || !V || !Qwin || !out_idx || !out_K || !out_V) return MMSHIFT_ERR_INVALID_ARG;
+  P.use_umma = choose_umma(P, K);
+  P.part_slots = P.use_umma ? kUmmaPartSlots : 1;
+  Buffers bf;
+  if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
+  bf.proxies_in = proxies_in;
+  bf.stats_in = stats_in;
+  if (dbg) {
+    bf.proxies_out = dbg->proxies;
+    if (dbg->group_mass && P.G) bf.gmass = dbg->group_mass;
+    if (dbg->anchor) bf.anchor = dbg->anchor;
+    if (dbg->scores) bf.scores = dbg->scores;
+    bf.mass = dbg->mass;
+  }
+  const cudaStream_t cs = (cudaStream_t)stream;
+  const StageMarks mk = marks_of(dbg, cs);
+  if ((st = run_mass(P, bf, K, Qwin, cs, mk)) != MMSHIFT_OK) return st;
+  cudaError_t e = mk.mark(5);
+  if (e == cudaSuccess && P.mode == MMSHIFT_SCORE_VOTE) e = launch_cover(P, bf, cs);
+  if (e == cudaSuccess) e = mk.mark(6);
+  if (e == cudaSuccess) e = launch_topk(P, bf, cs, out_idx, false);
+  if (e == cudaSuccess) e = mk.mark(7);
+  if (e == cudaSuccess) e = launch_gather(P, bf, cs, K, V, out_idx, out_K, out_V);
+  if (e == cudaSuccess) e = mk.mark(8);
+  if (dbg) {
+    const_cast<mmshift_debug*>(dbg)->launches = count_launches(P, bf);
+    const_cast<mmshift_debug*>(dbg)->score_path = P.use_umma ? 1 : 0;
+  }
+  return e == cudaSuccess ? MMSHIFT_OK : cuda_fail(e);
+}
+
 extern "C" {
 
 void mmshift_default_params(mmshift_params* p) {
@@ -269,6 +334,48 @@ mmshift_status mmshift_workspace_size(const mmshift_shape* s, const mmshift_para
   if (st != MMSHIFT_OK) return st;
   *bytes = layout_of(P).total;
   return MMSHIFT_OK;
+}
+
+
+mmshift_status mmshift_prefill_stats_workspace_size(const mmshift_shape* s, size_t* bytes) {
+  if (!bytes) return MMSHIFT_ERR_INVALID_ARG;
+  StatsJob J;
+  const mmshift_status st = stats_job(s, 0, &J);
+  if (st != MMSHIFT_OK) return st;
+  *bytes = align256((size_t)J.L * J.B * J.nchunk * 3 * J.ncol * sizeof(float));
+  return MMSHIFT_OK;
+}
+
+mmshift_status mmshift_prefill_stats(const mmshift_shape* s, const void* Qfull,
+                                     int64_t qfull_layer_stride, float* stats, void* workspace,
+                                     size_t workspace_bytes, mmshift_stream_t stream) {
+  StatsJob J;
+  mmshift_status st = stats_job(s, qfull_layer_stride, &J);
+  if (st != MMSHIFT_OK) return st;
+  if (!Qfull || !stats || !workspace) return MMSHIFT_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(Qfull) & 15) return MMSHIFT_ERR_INVALID_ARG;
+  size_t need = 0;
+  if ((st = mmshift_prefill_stats_workspace_size(s, &need)) != MMSHIFT_OK) return st;
+  if (workspace_bytes < need) return MMSHIFT_ERR_WORKSPACE;
+  const cudaError_t e = launch_prefill_stats(J, Qfull, static_cast<float*>(workspace), stats,
+                                             (cudaStream_t)stream, s->dtype == MMSHIFT_BF16);
+  return e == cudaSuccess ? MMSHIFT_OK : cuda_fail(e);
+}
+
+mmshift_status mmshift_build_proxies_from_stats(const mmshift_shape* s, const float* stats,
+                                                const mmshift_params* p, void* proxies,
+                                                mmshift_stream_t stream) {
+  Problem P;
+  mmshift_status st = prepare(s, p, &P);
+  if (st != MMSHIFT_OK) return st;
+  if (!p || !stats || !proxies) return MMSHIFT_ERR_INVALID_ARG;
+  if (P.Np == 0) return MMSHIFT_OK;
+  Buffers bf;
+  std::memset(&bf, 0, sizeof(bf));
+  bf.proxies_out = proxies;
+  bf.stats_in = stats;
+  const cudaError_t e = launch_proxy_pack(P, bf, (cudaStream_t)stream, nullptr);
+  return e == cudaSuccess ? MMSHIFT_OK : cuda_fail(e);
 }
 
 mmshift_status mmshift_build_proxies(const mmshift_shape* s, const void* Qwin,
@@ -360,37 +467,18 @@ mmshift_status mmshift_select(const mmshift_shape* s, const void* K, const void*
                               const mmshift_params* p, int32_t* out_idx, void* out_K,
                               void* out_V, const mmshift_debug* dbg, void* workspace,
                               size_t workspace_bytes, mmshift_stream_t stream) {
-  Problem P;
-  mmshift_status st = prepare(s, p, &P);
-  if (st != MMSHIFT_OK) return st;
-  if (!p || !K || !V || !Qwin || !out_idx || !out_K || !out_V) return MMSHIFT_ERR_INVALID_ARG;
-  P.use_umma = choose_umma(P, K);
-  P.part_slots = P.use_umma ? kUmmaPartSlots : 1;
-  Buffers bf;
-  if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
-  bf.proxies_in = proxies_in;
-  if (dbg) {
-    bf.proxies_out = dbg->proxies;
-    if (dbg->group_mass && P.G) bf.gmass = dbg->group_mass;
-    if (dbg->anchor) bf.anchor = dbg->anchor;
-    if (dbg->scores) bf.scores = dbg->scores;
-    bf.mass = dbg->mass;
-  }
-  const cudaStream_t cs = (cudaStream_t)stream;
-  const StageMarks mk = marks_of(dbg, cs);
-  if ((st = run_mass(P, bf, K, Qwin, cs, mk)) != MMSHIFT_OK) return st;
-  cudaError_t e = mk.mark(5);
-  if (e == cudaSuccess && P.mode == MMSHIFT_SCORE_VOTE) e = launch_cover(P, bf, cs);
-  if (e == cudaSuccess) e = mk.mark(6);
-  if (e == cudaSuccess) e = launch_topk(P, bf, cs, out_idx, false);
-  if (e == cudaSuccess) e = mk.mark(7);
-  if (e == cudaSuccess) e = launch_gather(P, bf, cs, K, V, out_idx, out_K, out_V);
-  if (e == cudaSuccess) e = mk.mark(8);
-  if (dbg) {
-    const_cast<mmshift_debug*>(dbg)->launches = count_launches(P, bf);
-    const_cast<mmshift_debug*>(dbg)->score_path = P.use_umma ? 1 : 0;
-  }
-  return e == cudaSuccess ? MMSHIFT_OK : cuda_fail(e);
+  return select_impl(s, K, V, Qwin, proxies_in, nullptr, p, out_idx, out_K, out_V, dbg,
+                     workspace, workspace_bytes, stream);
+}
+
+mmshift_status mmshift_select_with_stats(const mmshift_shape* s, const void* K, const void* V,
+                                         const void* Qwin, const float* stats,
+                                         const mmshift_params* p, int32_t* out_idx, void* out_K,
+                                         void* out_V, const mmshift_debug* dbg, void* workspace,
+                                         size_t workspace_bytes, mmshift_stream_t stream) {
+  if (!stats) return MMSHIFT_ERR_INVALID_ARG;
+  return select_impl(s, K, V, Qwin, nullptr, stats, p, out_idx, out_K, out_V, dbg, workspace,
+                     workspace_bytes, stream);
 }
 
 mmshift_status mmshift_poll_status(void* workspace, mmshift_stream_t stream) {

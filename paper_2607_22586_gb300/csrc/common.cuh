@@ -67,6 +67,16 @@ struct Buffers {
   float* mass;        // [L][Hkv][T] or null
   void* proxies_out;  // [L][B][Hq][Np][d] or null
   const void* proxies_in; // [L][B][Hq][Np][d] or null
+  const float* stats_in;  // [L][B][2][Hq][d] mean / std of the proxies, or null (window's)
+};
+
+// Whole-prefill statistics job (stats.cu).
+constexpr int kStatsChunk = 512;   // prompt queries per partial
+struct StatsJob {
+  int32_t L, B, ncol, nchunk;        // ncol = Hq * d; nchunk = max chunks per request
+  int64_t ls;                        // elements between layers of Q
+  int32_t t_len[MMSHIFT_MAX_BATCH];
+  int32_t tok_off[MMSHIFT_MAX_BATCH];
 };
 
 // Row p of the packed proxy block of KV head h: which group / query head /
@@ -125,6 +135,8 @@ __device__ __forceinline__ void set_status(int* status, int bit) {
 }
 
 // Host-side launchers (one translation unit each).
+cudaError_t launch_prefill_stats(const StatsJob& J, const void* Q, float* part, float* stats,
+                                 cudaStream_t st, bool bf16);
 cudaError_t launch_proxy_pack(const Problem& P, const Buffers& bf, cudaStream_t st,
                               const void* qwin);
 // ev (nullable): stage events 1 (softmax pass), 2 (merge) and 3 (mass pass)

@@ -136,9 +136,16 @@ __global__ void __launch_bounds__(256) proxy_pack_kernel(Problem P, Buffers bf, 
   __shared__ float mu[D], sg[D], rc[D / 2], rs[D / 2];
   constexpr int RPT = 256 / D;               // threads per dimension
   __shared__ float part[RPT][D];
-  const T* q = qwin + (size_t)l * P.ls_q + ((size_t)b * P.W * P.Hq + hq) * D;
+  const T* q = qwin ? qwin + (size_t)l * P.ls_q + ((size_t)b * P.W * P.Hq + hq) * D : nullptr;
   const size_t qstride = (size_t)P.Hq * D;
-  {
+  if (bf.stats_in) {
+    // given statistics (e.g. over the whole prefill): [L][B][2][Hq][D]
+    const float* st = bf.stats_in + (((size_t)l * P.B + b) * 2 * P.Hq + hq) * D;
+    for (int k = threadIdx.x; k < D; k += blockDim.x) {
+      mu[k] = st[k];
+      sg[k] = st[(size_t)P.Hq * D + k];
+    }
+  } else {
     // mean and unbiased std over the W window rows: thread (k, rg) sums rows
     // rg, rg + RPT, ... of dimension k; loads are independent and unrolled
     const int k = threadIdx.x % D, rg = threadIdx.x / D;

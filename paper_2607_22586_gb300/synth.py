@@ -214,6 +214,35 @@ def make_layer(wl: Workload, layer: int) -> LayerInputs:
     return LayerInputs(K=np.concatenate(ks), V=np.concatenate(vs), Qwin=np.stack(qs))
 
 
+def make_prompt_queries(wl: Workload, layer: int, li: LayerInputs,
+                        seed_tag: int = 0x51465550) -> np.ndarray:
+    """All prompt queries of one layer, [total_T, Hq, d] (dtype-exact float32),
+    consistent with ``li`` (the layer drawn by make_layer).
+
+    Text positions follow the window recipe (half the request's per-head key
+    mean plus unit normal noise); visual positions add a seeded per-(head,
+    dimension) modality offset drawn N(0, 1) per request, so that prompt-wide
+    and window statistics differ the way text and image tokens do. The last
+    min(W, T) rows of each request are its window queries ``li.Qwin``.
+    """
+    rng = np.random.Generator(np.random.Philox(key=[wl.seed ^ seed_tag, layer]))
+    hq, hkv, d, w = wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.window
+    r = hq // hkv
+    cu = wl.cu_seqlens()
+    out = np.empty((wl.total_tokens, hq, d), dtype=np.float32)
+    for b, (t_len, n_vis) in enumerate(zip(wl.seq_lens, wl.n_visual)):
+        k = li.K[cu[b]:cu[b + 1]]
+        kmean = k.mean(axis=0, dtype=np.float64).astype(np.float32)
+        q = (np.float32(0.5) * np.repeat(kmean, r, axis=0)[None, :, :]
+             + rng.standard_normal((t_len, hq, d), dtype=np.float32))
+        q[:n_vis] += rng.standard_normal((hq, d), dtype=np.float32)[None]
+        q = round_to_dtype(q, wl.dtype)
+        nw = min(w, t_len)
+        q[t_len - nw:] = li.Qwin[b, w - nw:]
+        out[cu[b]:cu[b + 1]] = q
+    return out
+
+
 def make_proxies(wl: Workload, n_proxies: int, layer: int, scale: float = 8.0,
                  seed_tag: int = 0x50524F58) -> np.ndarray:
     """Seeded stand-alone proxy set [B, Hq, N_p, d] (dtype-exact float32).

@@ -79,16 +79,20 @@ def shape_of(wl: S.Workload, n_layers: int = 1, window=None):
                         layer_stride_q=wl.batch * w * wl.n_q_heads * wl.head_dim)
 
 
-def gpu_select(wl: S.Workload, layers, h, proxies=None):
+def gpu_select(wl: S.Workload, layers, h, proxies=None, stats=None):
     """Run mmshift_select over ``layers`` (list of LayerInputs) in one call
-    with every debug output; returns numpy arrays [L, ...]."""
+    with every debug output (mmshift_select_with_stats when ``stats``, a
+    device tensor [L, B, 2, Hq*d], is given); returns numpy arrays [L, ...]."""
     L = len(layers)
     shape = shape_of(wl, L)
     params = abi_params(h)
     K = dev(np.stack([li.K for li in layers]), wl.dtype)
     V = dev(np.stack([li.V for li in layers]), wl.dtype)
     Q = dev(np.stack([li.Qwin for li in layers]), wl.dtype)
-    pin = dev(proxies, wl.dtype) if proxies is not None else None
+    if proxies is None or isinstance(proxies, torch.Tensor):
+        pin = proxies
+    else:
+        pin = dev(proxies, wl.dtype)
     rows = M.mmshift_output_rows(shape)
     ws_bytes = M.mmshift_workspace_size(shape, params)
     ws = torch.zeros(ws_bytes, dtype=torch.uint8, device="cuda")
@@ -103,7 +107,11 @@ def gpu_select(wl: S.Workload, layers, h, proxies=None):
     sc = torch.full((L, hkv, T), -1.0, device="cuda")
     px = torch.empty((L, wl.batch, hq, max(h["n_proxies"], 1), d), dtype=TORCH_DT[wl.dtype], device="cuda")
     dbg = M.make_debug(proxies=px, group_mass=gm, anchor=an, mass=ms, scores=sc)
-    st = M.mmshift_select(shape, K, V, Q, pin, params, out_idx, out_k, out_v, dbg, ws, ws_bytes)
+    if stats is None:
+        st = M.mmshift_select(shape, K, V, Q, pin, params, out_idx, out_k, out_v, dbg, ws, ws_bytes)
+    else:
+        st = M.mmshift_select_with_stats(shape, K, V, Q, stats, params, out_idx, out_k, out_v, dbg,
+                                         ws, ws_bytes)
     M.check(st, "mmshift_select")
     M.check(M.mmshift_poll_status(ws), "mmshift_poll_status")
     torch.cuda.synchronize()

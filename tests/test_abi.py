@@ -93,3 +93,20 @@ def test_null_and_workspace_errors_return_before_any_launch():
     assert M.mmshift_gather(s, fake, fake, None, fake, fake, fake, n) == L.MMSHIFT_ERR_INVALID_ARG
     lib = M.load_library()
     assert lib.mmshift_status_string(L.MMSHIFT_ERR_TIMEOUT) == b"device-side wait timed out"
+
+
+def test_prefill_stats_validation_before_any_launch():
+    s = _shape()
+    n = M.mmshift_prefill_stats_workspace_size(s)
+    # per layer and request: ceil(T / 512) chunks x 3 partial sums x Hq * d floats
+    assert n == ((1 * 2 * 1 * 3 * 8 * 128 * 4 + 255) // 256) * 256
+    fake = 1 << 40
+    assert M.mmshift_prefill_stats(s, None, 0, fake, fake, n) == L.MMSHIFT_ERR_INVALID_ARG
+    assert M.mmshift_prefill_stats(s, fake + 4, 0, fake, fake, n) == L.MMSHIFT_ERR_INVALID_ARG  # unaligned
+    assert M.mmshift_prefill_stats(s, fake, 0, fake, fake, n - 256) == L.MMSHIFT_ERR_WORKSPACE
+    assert M.mmshift_prefill_stats(s, fake, 12, fake, fake, n) == L.MMSHIFT_ERR_INVALID_ARG  # stride
+    s2 = _shape(n_layers=2, layer_stride_kv=250 * 2 * 128, layer_stride_q=2 * 8 * 8 * 128)
+    assert M.mmshift_prefill_stats(s2, fake, 100, fake, fake, n) == L.MMSHIFT_ERR_INVALID_ARG  # too small
+    p = M.default_params()
+    assert M.mmshift_build_proxies_from_stats(s, None, p, fake) == L.MMSHIFT_ERR_INVALID_ARG
+    assert M.mmshift_build_proxies_from_stats(s, fake, p, None) == L.MMSHIFT_ERR_INVALID_ARG
