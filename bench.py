@@ -55,6 +55,12 @@ SFU_EX2_PER_SM_CLK = 32          # MUFU.EX2 lanes per SM per clock on GB300 (mea
 SCORE_TRAFFIC = {"source_sha256_16": "dc3a01adad94c3e9", "workload": "qwen7b-28l-32k",
                  "proxies": "paper", "softmax_pass": 7 * (154.181632e6 + 44.690176e6),
                  "mass_pass": 7 * (156.648704e6 + 46.562816e6)}
+# DRAM traffic of the prompt-query statistics pass (both kernels) per launch
+# of the default workload, from one ncu capture of a 4-layer slice scaled by 7
+# (partial kernel 939.590912 MB read + 3.059712 MB written, merge 11.026176 MB
+# read); valid for the stats.cu it was measured on (checked by hash).
+STATS_TRAFFIC = {"source_sha256_16": "ddcbfa1963474036", "workload": "qwen7b-28l-32k",
+                 "bytes": 7 * (939.590912e6 + 3.059712e6 + 11.026176e6)}
 UNIT = "tokens/s/layer"
 SM_COUNT = 152
 FP32_LANES_PER_SM = 128
@@ -224,16 +230,28 @@ def algorithmic(wl, hyper):
     return k_read + gather, k_read, pass_flops
 
 
+def _source_digest(name):
+    import hashlib
+    try:
+        with open(os.path.join(ROOT, "paper_2607_22586_gb300", "csrc", name), "rb") as f:
+            return hashlib.sha256(f.read()).hexdigest()[:16]
+    except OSError:
+        return None
+
+
+def stats_traffic(wl):
+    """DRAM bytes per launch of the statistics pass from the recorded capture,
+    or None if stats.cu or the workload differ from the captured ones."""
+    t = STATS_TRAFFIC
+    if _source_digest("stats.cu") != t["source_sha256_16"] or wl.name != t["workload"]:
+        return None
+    return t["bytes"]
+
+
 def score_traffic(wl, args, kernel):
     """DRAM bytes per launch of a scoring kernel from the recorded capture, or
     None if the kernel source or the workload differ from the captured ones."""
-    import hashlib
-    src = os.path.join(ROOT, "paper_2607_22586_gb300", "csrc", "score_umma.cu")
-    try:
-        with open(src, "rb") as f:
-            digest = hashlib.sha256(f.read()).hexdigest()[:16]
-    except OSError:
-        return None
+    digest = _source_digest("score_umma.cu")
     t = SCORE_TRAFFIC
     if digest != t["source_sha256_16"] or wl.name != t["workload"] or args.proxies != t["proxies"]:
         return None
@@ -483,7 +501,7 @@ def run_gpu(args, wl):
         st_ms = stage_ms["prefill_stats"]
         ach = s_bytes / (st_ms * 1e-3) / 1e9
         stats_roof = {"bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                      "frac": ach / peaks["hbm_gbs"], "traffic": None,
+                      "frac": ach / peaks["hbm_gbs"], "traffic": stats_traffic(wl),
                       "kernel": "stats_partial_kernel + stats_merge_kernel",
                       "bytes_per_launch": s_bytes, "peak_kind": f"HBM copy ({peak_src})"}
     tokens_layer = T * L * world          # metric unit: tokens per second per layer

@@ -9,7 +9,7 @@
 //    one request and layer, one thread per 8 consecutive columns (q-head,
 //    dimension) up to 1024 threads; a thread keeps, per column, the sums of
 //    (x - x0) and (x - x0)^2 in fp32, x0 being the chunk's first query (the
-//    shift keeps the second sum free of cancellation), with four rows' loads
+//    shift keeps the second sum free of cancellation), with eight rows' loads
 //    in flight.
 //  - stats_merge_kernel: one thread per column merges the chunks in order with
 //    the pairwise update of Chan, Golub and LeVeque (count, mean, sum of
@@ -20,6 +20,9 @@
 
 namespace mmshift {
 namespace {
+
+constexpr int kStatsRows = 8;      // rows of loads in flight per thread
+constexpr int kMergeAhead = 8;     // chunks of partial sums loaded ahead in the merge
 
 template <typename T>
 __device__ __forceinline__ void load8(const T* p, float (&x)[8]);
@@ -58,13 +61,13 @@ __global__ void __launch_bounds__(1024) stats_partial_kernel(StatsJob J, const T
 #pragma unroll
     for (int k = 0; k < 8; ++k) { s1[k] = 0.f; s2[k] = 0.f; }
     int t = 1;
-    // four independent rows in flight
-    for (; t + 4 <= t1 - t0; t += 4) {
-      float x[4][8];
+    // kStatsRows independent rows in flight
+    for (; t + kStatsRows <= t1 - t0; t += kStatsRows) {
+      float x[kStatsRows][8];
 #pragma unroll
-      for (int u = 0; u < 4; ++u) load8(col + (size_t)(t + u) * J.ncol, x[u]);
+      for (int u = 0; u < kStatsRows; ++u) load8(col + (size_t)(t + u) * J.ncol, x[u]);
 #pragma unroll
-      for (int u = 0; u < 4; ++u)
+      for (int u = 0; u < kStatsRows; ++u)
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
           const float dv = x[u][k] - x0[k];
@@ -101,18 +104,28 @@ __global__ void __launch_bounds__(256) stats_merge_kernel(StatsJob J, const floa
   const float* in = part + ((size_t)l * J.B + b) * J.nchunk * 3 * J.ncol + col;
   float n = 0.f, mean = 0.f, m2 = 0.f;
   const int nch = (t_len + kStatsChunk - 1) / kStatsChunk;
-  for (int c = 0; c < nch; ++c) {
-    const float nb = (float)(min(t_len, (c + 1) * kStatsChunk) - c * kStatsChunk);
-    const float x0 = in[(size_t)c * 3 * J.ncol];
-    const float s1 = in[((size_t)c * 3 + 1) * J.ncol];
-    const float s2 = in[((size_t)c * 3 + 2) * J.ncol];
-    const float mb = x0 + s1 / nb;
-    const float m2b = fmaxf(s2 - s1 * (s1 / nb), 0.f);
-    const float nab = n + nb;
-    const float delta = mb - mean;
-    mean += delta * (nb / nab);
-    m2 += m2b + delta * delta * (n * nb / nab);
-    n = nab;
+  for (int c0 = 0; c0 < nch; c0 += kMergeAhead) {
+    // the loads of kMergeAhead chunks first, then the merges in chunk order
+    float v[kMergeAhead][3];
+#pragma unroll
+    for (int u = 0; u < kMergeAhead; ++u)
+      if (c0 + u < nch)
+#pragma unroll
+        for (int q = 0; q < 3; ++q) v[u][q] = in[((size_t)(c0 + u) * 3 + q) * J.ncol];
+#pragma unroll
+    for (int u = 0; u < kMergeAhead; ++u) {
+      const int c = c0 + u;
+      if (c >= nch) break;
+      const float nb = (float)(min(t_len, (c + 1) * kStatsChunk) - c * kStatsChunk);
+      const float x0 = v[u][0], s1 = v[u][1], s2 = v[u][2];
+      const float mb = x0 + s1 / nb;
+      const float m2b = fmaxf(s2 - s1 * (s1 / nb), 0.f);
+      const float nab = n + nb;
+      const float delta = mb - mean;
+      mean += delta * (nb / nab);
+      m2 += m2b + delta * delta * (n * nb / nab);
+      n = nab;
+    }
   }
   float* out = stats + ((size_t)l * J.B + b) * 2 * J.ncol;
   out[col] = mean;
