@@ -32,7 +32,7 @@ F32 = "f32"
 __all__ = [
     "DEFAULTS", "SCORE_VOTE", "SCORE_MASS", "BF16", "F32", "philox4x64_10", "uniforms_from_bits",
     "proxy_normals", "window_stats", "prefill_stats", "rope_rotate", "round_to",
-    "build_proxies", "build_proxies_from_stats",
+    "build_proxies", "build_proxies_from_stats", "hidden_normals", "hidden_proxies",
     "softmax_rows", "group_masses", "anchor_attention", "cover_sets", "votes",
     "scores", "select_topk", "gather", "select_request", "select",
 ]
@@ -92,12 +92,13 @@ def uniforms_from_bits(x: np.ndarray) -> np.ndarray:
 
 
 def proxy_normals(seed: int, layer_id: int, b: int, n_q_heads: int,
-                  n_proxies: int, head_dim: int) -> np.ndarray:
+                  n_proxies: int, head_dim: int, stream: int = 0) -> np.ndarray:
     """Standard normals z[hq, i, j] for request b of layer ``layer_id``.
 
     One Philox4x64-10 draw with counter (i * d/8 + q, hq, b, layer_id) and key
-    (seed, 0) covers dims 4q..4q+3 and d/2+4q..d/2+4q+3 of proxy i of query
-    head hq. Its four 64-bit outputs, split low word first, give eight 32-bit
+    (seed, stream) covers dims 4q..4q+3 and d/2+4q..d/2+4q+3 of proxy i of
+    query head hq (stream 0: query-space proxies; stream 1: hidden-space
+    proxies, see hidden_normals). Its four 64-bit outputs, split low word first, give eight 32-bit
     words w0..w7 and uniforms u_k = ((w_k >> 9) + 1/2) 2^-23; Box-Muller turns
     each pair (u_2m, u_2m+1) into sqrt(-2 ln u_2m) (cos, sin)(2 pi u_2m+1).
     Pairs 0, 1 fill dims 4q..4q+3; pairs 2, 3 fill d/2+4q..d/2+4q+3.
@@ -110,7 +111,7 @@ def proxy_normals(seed: int, layer_id: int, b: int, n_q_heads: int,
     ctr = np.stack([i * np.uint64(nq) + q, hq,
                     np.full_like(q, np.uint64(b)),
                     np.full_like(q, np.uint64(layer_id))], axis=-1)
-    x = philox4x64_10(ctr, (seed & 0xFFFFFFFFFFFFFFFF, 0))      # [Hq, Np, d/8, 4]
+    x = philox4x64_10(ctr, (seed & 0xFFFFFFFFFFFFFFFF, stream))  # [Hq, Np, d/8, 4]
     words = np.stack([x & _M32, x >> _S32], axis=-1).reshape(x.shape[:-1] + (8,))
     u = uniforms_from_bits(words)                               # [Hq, Np, d/8, 8]
     r = np.sqrt(-2.0 * np.log(u[..., 0::2]))                    # [.., 4]
@@ -152,7 +153,9 @@ def prefill_stats(qfull: np.ndarray):
 
     Reading: in query space, per (query head, dimension) over all T prompt
     queries of the request, with the unbiased (T - 1) estimator (0 for T = 1).
-    qfull: [T, Hq, d] -> (mu, sigma), each [Hq, d] float64.
+    qfull: [T, Hq, d] -> (mu, sigma), each [Hq, d] float64. The same
+    statistics of hidden states [T, d_model] (the paper's own space) give
+    [d_model] vectors for hidden_proxies.
     """
     q = np.asarray(qfull, dtype=np.float64)
     t = q.shape[0]
@@ -216,6 +219,46 @@ def build_proxies_from_stats(mu: np.ndarray, sigma: np.ndarray, z: np.ndarray, g
     q = mu[:, None, :] + gamma * sigma[:, None, :] * z
     if rope_theta > 0.0:
         q = rope_rotate(q, float(t_len + rope_pos_offset), rope_theta)
+    return round_to(q, dtype)
+
+
+def hidden_normals(seed: int, layer_id: int, b: int, n_proxies: int, d_model: int) -> np.ndarray:
+    """Standard normals z[i, j] of the N proxy hidden states of request b
+    (§3.2.1: H~_i ~ N(mu_pre, diag((gamma sigma_pre)^2)) in the model's
+    hidden space). Reading: the generator of proxy_normals with key
+    (seed, 1) and one 'head' of width d_model: counter
+    (i * d_model/8 + q, 0, b, layer_id) covers dims 4q..4q+3 and
+    d_model/2+4q..d_model/2+4q+3. -> [N, d_model] float64.
+    """
+    return proxy_normals(seed, layer_id, b, 1, n_proxies, d_model, stream=1)[0]
+
+
+def hidden_proxies(mu: np.ndarray, sigma: np.ndarray, z: np.ndarray, w_q: np.ndarray,
+                   bias: Optional[np.ndarray], gamma: float, n_q_heads: int, pos: float,
+                   dtype: str, rope_theta: float = 0.0) -> np.ndarray:
+    """Query proxies from proxy hidden states (§3.2.1, Algorithm 1's first
+    steps): H~_i = mu + gamma * sigma * z_i in the hidden space, projected by
+    the query projection q~_i^(h) = W_Q^(h) H~_i, then placed at a future
+    position with RoPE.
+
+    mu, sigma: [d_model] statistics of the prefill hidden states
+    (prefill_stats over [T, d_model]); z: [N, d_model] (hidden_normals);
+    w_q: [Hq*d, d_model] (row f of the projection gives output feature f =
+    hq*d + j); bias: [Hq*d] or None; pos: the proxies' position.
+    Reading: H~ is rounded to the input dtype before the projection (the
+    model's projection consumes hidden states in that dtype); the projection,
+    the bias (Qwen-style query projections carry one) and RoPE are exact
+    (float64) and the proxies are rounded once at the end, as in
+    build_proxies. -> [Hq, N, d] float64 (dtype-exact).
+    """
+    h = round_to(mu[None, :] + gamma * sigma[None, :] * z, dtype)      # [N, d_model]
+    q = h @ np.asarray(w_q, dtype=np.float64).T                        # [N, Hq*d]
+    if bias is not None:
+        q = q + np.asarray(bias, dtype=np.float64)[None, :]
+    n = q.shape[0]
+    q = q.reshape(n, n_q_heads, -1).transpose(1, 0, 2)                 # [Hq, N, d]
+    if rope_theta > 0.0:
+        q = rope_rotate(q, float(pos), rope_theta)
     return round_to(q, dtype)
 
 

@@ -126,6 +126,37 @@ def _philox_9_rounds(ctr, key):
     return np.stack(c, axis=-1)
 
 
+def _hidden_proxies_transposed(mu, sigma, z, w_q, bias, gamma, n_q_heads, pos, dtype,
+                               rope_theta=0.0):
+    h = O.round_to(mu[None, :] + gamma * sigma[None, :] * z, dtype)
+    q = h @ np.asarray(w_q, dtype=np.float64)
+    if bias is not None:
+        q = q + bias[None, :]
+    q = q.reshape(q.shape[0], n_q_heads, -1).transpose(1, 0, 2)
+    return O.round_to(q, dtype)
+
+
+def _hidden_proxies_no_bias(mu, sigma, z, w_q, bias, gamma, n_q_heads, pos, dtype, rope_theta=0.0):
+    h = O.round_to(mu[None, :] + gamma * sigma[None, :] * z, dtype)
+    q = (h @ np.asarray(w_q, dtype=np.float64).T)
+    q = q.reshape(q.shape[0], n_q_heads, -1).transpose(1, 0, 2)
+    return O.round_to(q, dtype)
+
+
+def _hidden_proxies_unrounded_hidden(mu, sigma, z, w_q, bias, gamma, n_q_heads, pos, dtype,
+                                     rope_theta=0.0):
+    h = mu[None, :] + gamma * sigma[None, :] * z
+    q = h @ np.asarray(w_q, dtype=np.float64).T
+    if bias is not None:
+        q = q + bias[None, :]
+    q = q.reshape(q.shape[0], n_q_heads, -1).transpose(1, 0, 2)
+    return O.round_to(q, dtype)
+
+
+def _hidden_normals_query_stream(seed, layer_id, b, n_proxies, d_model):
+    return O.proxy_normals(seed, layer_id, b, 1, n_proxies, d_model)[0]
+
+
 MUTANTS = {
     "std_ddof0": ("window_stats", _window_stats_ddof0),
     "prefill_std_ddof0": ("prefill_stats", _prefill_stats_ddof0),
@@ -142,6 +173,10 @@ MUTANTS = {
     "rope_sign": ("rope_rotate", _rope_wrong_sign),
     "bf16_truncation": ("round_to", _round_truncate),
     "philox_9_rounds": ("philox4x64_10", _philox_9_rounds),
+    "hidden_projection_transposed": ("hidden_proxies", _hidden_proxies_transposed),
+    "hidden_projection_no_bias": ("hidden_proxies", _hidden_proxies_no_bias),
+    "hidden_states_not_rounded": ("hidden_proxies", _hidden_proxies_unrounded_hidden),
+    "hidden_normals_query_stream": ("hidden_normals", _hidden_normals_query_stream),
 }
 
 

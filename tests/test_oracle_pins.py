@@ -96,6 +96,55 @@ def pin_prefill_stats(orc=O):
     assert np.array_equal(w, orc.build_proxies_from_stats(m, sg, z, 3.0, 50, orc.BF16))
 
 
+def pin_hidden_proxies(orc=O):
+    """§3.2.1 hidden-space proxies q~ = W_Q (mu + gamma sigma z) (+ bias):
+    an identity projection reduces them to the query-space expansion; the
+    proxies' mean and covariance follow W_Q mu + b and
+    gamma^2 W_Q diag(sigma^2) W_Q^T (a non-symmetric W_Q, so a transposed
+    operand fails); a difference of two hidden dims below half a bf16 ulp
+    survives only if the hidden proxies are rounded before the projection;
+    the hidden stream is Philox with key (seed, 1)."""
+    rng = np.random.default_rng(31)
+    hq, d, n = 3, 8, 40
+    dm = hq * d
+    mu = rng.normal(size=dm)
+    sig = rng.uniform(0.2, 1.5, size=dm)
+    z = orc.hidden_normals(seed=9, layer_id=2, b=1, n_proxies=n, d_model=dm)
+    got = orc.hidden_proxies(mu, sig, z, np.eye(dm), None, 4.0, hq, 0.0, orc.BF16)
+    ref = orc.build_proxies_from_stats(mu.reshape(hq, d), sig.reshape(hq, d),
+                                       z.reshape(n, hq, d).transpose(1, 0, 2), 4.0, 100, orc.BF16)
+    assert np.array_equal(got, ref)
+    # moments over many proxies (float32: rounding far below the CLT band)
+    dm, n, gamma = 8, 1 << 15, 2.0
+    mu = np.array([0.3, -1.0, 2.0, 0.0, 0.5, -0.25, 1.5, -0.75])
+    sig = np.array([0.5, 1.0, 0.25, 2.0, 0.75, 1.25, 0.1, 0.6])
+    w = rng.normal(size=(dm, dm))
+    bias = rng.normal(size=dm)
+    z = orc.hidden_normals(seed=4, layer_id=0, b=0, n_proxies=n, d_model=dm)
+    q = orc.hidden_proxies(mu, sig, z, w, bias, gamma, 1, 0.0, orc.F32)[0]   # [N, dm]
+    mean_ref = w @ mu + bias
+    cov_ref = gamma ** 2 * w @ np.diag(sig ** 2) @ w.T
+    sd = np.sqrt(np.diag(cov_ref))
+    assert np.all(np.abs(q.mean(axis=0) - mean_ref) < 6.0 * sd / math.sqrt(n))
+    cov = np.cov(q.T)
+    assert np.all(np.abs(cov - cov_ref) < 8.0 * np.outer(sd, sd) / math.sqrt(n))
+    # rounding of H~ before the projection
+    mu = np.zeros(8)
+    mu[:2] = [1.0 + 0.49 * 2.0 ** -7, 1.0]
+    w = np.zeros((8, 8))
+    w[0, :2] = [1.0, -1.0]
+    q = orc.hidden_proxies(mu, np.zeros(8), np.zeros((1, 8)), w, None, 1.0, 1, 0.0, orc.BF16)
+    assert q.shape == (1, 1, 8) and np.all(q == 0.0)
+    # the hidden stream is Philox with key (seed, 1)
+    # numpy advances the counter before a block: counter (2, 0, 3, 7) is proxy 0, quad 2
+    x = np.random.Philox(key=[5, 1], counter=[1, 0, 3, 7]).random_raw(4)
+    w32 = np.stack([x & 0xFFFFFFFF, x >> 32], axis=-1).reshape(-1)
+    u = orc.uniforms_from_bits(w32)
+    zz = np.sqrt(-2.0 * np.log(u[0::2])) * np.cos(2.0 * np.pi * u[1::2])
+    z = orc.hidden_normals(seed=5, layer_id=7, b=3, n_proxies=1, d_model=64)
+    assert math.isclose(z[0, 4 * 2], zz[0], rel_tol=1e-12)
+
+
 def pin_sampler_closed_form(orc=O):
     """Appendix A.2: for q ~ N(mu, Sigma), E[exp(q.k/sqrt d)] =
     exp(mu.k/sqrt d + k^T Sigma k / (2d)). With Sigma = diag((gamma*sigma)^2)
@@ -317,6 +366,7 @@ def pin_topk_bruteforce(orc=O):
 
 
 ALL_PINS = [pin_philox_vs_numpy, pin_normals_distribution, pin_window_stats, pin_prefill_stats,
+            pin_hidden_proxies,
             pin_sampler_closed_form, pin_rope, pin_round_bf16, pin_mass_totals,
             pin_sigma_zero_single_query, pin_shift_and_permutation, pin_budget_ge_t,
             pin_lastattn, pin_uniform_keys, pin_cover_bruteforce, pin_topk_bruteforce]
