@@ -169,6 +169,48 @@ mmshift_status mmshift_prefill_stats(const mmshift_shape* s, const void* Qfull,
                                      int64_t qfull_layer_stride, float* stats, void* workspace,
                                      size_t workspace_bytes, mmshift_stream_t stream);
 
+/* Hidden-state statistics (Section 3.2.1: mu_pre, sigma_pre of the hidden
+ * states entering layer l, per feature over all T_b prompt tokens of
+ * request b, unbiased, 0 for T_b = 1): the reduction of mmshift_prefill_stats
+ * over d_model columns. H: [L][T_total][d_model] in the shape's dtype, layers
+ * `h_layer_stride` elements apart (0 = dense; a multiple of 8), 16-byte
+ * aligned; d_model a multiple of 8. stats: [L][batch][2][d_model] float32
+ * (mean, std). workspace: mmshift_hidden_stats_workspace_size() bytes. */
+mmshift_status mmshift_hidden_stats_workspace_size(const mmshift_shape* s, int32_t d_model,
+                                                  size_t* bytes);
+mmshift_status mmshift_hidden_stats(const mmshift_shape* s, int32_t d_model, const void* H,
+                                    int64_t h_layer_stride, float* stats, void* workspace,
+                                    size_t workspace_bytes, mmshift_stream_t stream);
+
+/* Step 1 in the hidden space (Section 3.2.1, the paper's construction):
+ * N proxy hidden states H~_i = mu + gamma * sigma * z_i per (layer, request),
+ * z from Philox4x64-10 with key (seed, 1) and counter
+ * (i * d_model/8 + q, 0, b, layer_id + l) covering features [4q, 4q+4) and
+ * [d_model/2 + 4q, +4) (Box-Muller on consecutive uniforms), rounded to
+ * bf16, projected by the query projection on the tensor cores,
+ * q~_i = W_Q H~_i + b_Q (fp32 accumulation), rotated by RoPE (rotate-half
+ * pairs within each head, when params->rope_theta > 0) to position
+ * rope_pos[b] (host array, nullable: T_b + rope_pos_offset; for M-RoPE
+ * models pass the text position of the first decoded token, where the three
+ * M-RoPE components coincide) and rounded to bf16.
+ * hstats: [L][batch][2][d_model] float32 (mmshift_hidden_stats);
+ * W_Q: [L][Hq*d][d_model] bf16 (row hq*d + j = output feature j of query
+ * head hq), layers `wq_layer_stride` elements apart (0 = dense; a multiple
+ * of 8), 16-byte aligned; bias_q: [L][Hq*d] bf16 or NULL. proxies:
+ * [L, batch, Hq, N, d] bf16, for mmshift_select / mmshift_proxy_mass as
+ * `proxies_in`. workspace: mmshift_hidden_proxies_workspace_size() bytes,
+ * 256-byte aligned (its first word is the status mmshift_poll_status reads).
+ * bf16 only (MMSHIFT_ERR_UNSUPPORTED otherwise); d_model a multiple of 64,
+ * Hq*d a multiple of 128; needs the tensor-core path (sm_100 family). */
+mmshift_status mmshift_hidden_proxies_workspace_size(const mmshift_shape* s, int32_t d_model,
+                                                     const mmshift_params* p, size_t* bytes);
+mmshift_status mmshift_build_hidden_proxies(const mmshift_shape* s, int32_t d_model,
+                                            const float* hstats, const void* W_Q,
+                                            int64_t wq_layer_stride, const void* bias_q,
+                                            const int32_t* rope_pos, const mmshift_params* p,
+                                            void* proxies, void* workspace,
+                                            size_t workspace_bytes, mmshift_stream_t stream);
+
 /* Step 1 from given statistics (e.g. mmshift_prefill_stats) instead of the
  * observation window's: q~ = mu + gamma * sigma * z with the same normals,
  * RoPE and rounding as mmshift_build_proxies. stats: [L][batch][2][Hq][d]

@@ -12,4 +12,6 @@ from ._lib import (MMShiftError, Params, Shape, Debug, check, default_params,  #
                    mmshift_output_rows, mmshift_poll_status, mmshift_proxy_mass,
                    mmshift_scores_topk, mmshift_scores_topk_noalloc, mmshift_select, mmshift_topk,
                    mmshift_workspace_size, mmshift_prefill_stats, mmshift_prefill_stats_workspace_size,
-                   mmshift_build_proxies_from_stats, mmshift_select_with_stats)
+                   mmshift_build_proxies_from_stats, mmshift_select_with_stats,
+                   mmshift_hidden_stats_workspace_size, mmshift_hidden_stats,
+                   mmshift_hidden_proxies_workspace_size, mmshift_build_hidden_proxies)

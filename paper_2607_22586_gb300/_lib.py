@@ -34,6 +34,8 @@ EXPORTED = [
     "mmshift_last_cuda_error", "mmshift_scores_topk_noalloc",
     "mmshift_prefill_stats_workspace_size", "mmshift_prefill_stats",
     "mmshift_build_proxies_from_stats", "mmshift_select_with_stats",
+    "mmshift_hidden_stats_workspace_size", "mmshift_hidden_stats",
+    "mmshift_hidden_proxies_workspace_size", "mmshift_build_hidden_proxies",
 ]
 MMSHIFT_NOALLOC_SCRATCH_BYTES = 8 << 20
 
@@ -102,6 +104,17 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.mmshift_prefill_stats.restype = st
     lib.mmshift_build_proxies_from_stats.argtypes = [_SP, _VP, _PP, _VP, _VP]
     lib.mmshift_build_proxies_from_stats.restype = st
+    lib.mmshift_hidden_stats_workspace_size.argtypes = [_SP, ctypes.c_int32, ctypes.POINTER(ctypes.c_size_t)]
+    lib.mmshift_hidden_stats_workspace_size.restype = st
+    lib.mmshift_hidden_stats.argtypes = [_SP, ctypes.c_int32, _VP, ctypes.c_int64, _VP, _VP,
+                                         ctypes.c_size_t, _VP]
+    lib.mmshift_hidden_stats.restype = st
+    lib.mmshift_hidden_proxies_workspace_size.argtypes = [_SP, ctypes.c_int32, _PP,
+                                                          ctypes.POINTER(ctypes.c_size_t)]
+    lib.mmshift_hidden_proxies_workspace_size.restype = st
+    lib.mmshift_build_hidden_proxies.argtypes = [_SP, ctypes.c_int32, _VP, _VP, ctypes.c_int64, _VP,
+                                                 _VP, _PP, _VP, _VP, ctypes.c_size_t, _VP]
+    lib.mmshift_build_hidden_proxies.restype = st
     lib.mmshift_proxy_mass.argtypes = [_SP, _VP, _VP, _VP, _PP, _VP, _VP, _VP, _VP, ctypes.c_size_t, _VP]
     lib.mmshift_proxy_mass.restype = st
     lib.mmshift_scores_topk.argtypes = [_SP, _PP, _VP, _VP, _VP, _VP, _VP, ctypes.c_size_t, _VP]
@@ -205,6 +218,42 @@ def mmshift_prefill_stats(shape, qfull, qfull_layer_stride, stats, workspace, wo
     return load_library().mmshift_prefill_stats(ctypes.byref(shape), _ptr(qfull),
                                                 int(qfull_layer_stride), _ptr(stats),
                                                 _ptr(workspace), workspace_bytes, _ptr(stream))
+
+
+
+def mmshift_hidden_stats_workspace_size(shape: Shape, d_model: int) -> int:
+    n = ctypes.c_size_t()
+    check(load_library().mmshift_hidden_stats_workspace_size(ctypes.byref(shape), int(d_model),
+                                                             ctypes.byref(n)),
+          "mmshift_hidden_stats_workspace_size")
+    return n.value
+
+
+def mmshift_hidden_stats(shape, d_model, H, h_layer_stride, stats, workspace, workspace_bytes,
+                         stream=None) -> int:
+    return load_library().mmshift_hidden_stats(ctypes.byref(shape), int(d_model), _ptr(H),
+                                               int(h_layer_stride), _ptr(stats), _ptr(workspace),
+                                               workspace_bytes, _ptr(stream))
+
+
+def mmshift_hidden_proxies_workspace_size(shape: Shape, d_model: int, params) -> int:
+    n = ctypes.c_size_t()
+    check(load_library().mmshift_hidden_proxies_workspace_size(ctypes.byref(shape), int(d_model),
+                                                               ctypes.byref(params), ctypes.byref(n)),
+          "mmshift_hidden_proxies_workspace_size")
+    return n.value
+
+
+def mmshift_build_hidden_proxies(shape, d_model, hstats, W_Q, wq_layer_stride, bias_q, rope_pos,
+                                 params, proxies, workspace, workspace_bytes, stream=None) -> int:
+    """rope_pos: None or a sequence of per-request positions (host int32)."""
+    pos = None
+    if rope_pos is not None:
+        pos = (ctypes.c_int32 * len(rope_pos))(*[int(x) for x in rope_pos])
+    return load_library().mmshift_build_hidden_proxies(
+        ctypes.byref(shape), int(d_model), _ptr(hstats), _ptr(W_Q), int(wq_layer_stride),
+        _ptr(bias_q), pos, ctypes.byref(params), _ptr(proxies), _ptr(workspace), workspace_bytes,
+        _ptr(stream))
 
 
 def mmshift_build_proxies_from_stats(shape, stats, params, proxies, stream=None) -> int:

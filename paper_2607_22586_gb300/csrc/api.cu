@@ -234,13 +234,15 @@ mmshift_status noalloc_cuda_fail(cudaError_t e) { return cuda_fail(e); }
 }  // namespace mmshift
 
 // Whole-prefill statistics job of a shape (no hyper-parameters involved).
-static mmshift_status stats_job(const mmshift_shape* s, int64_t qfull_layer_stride, StatsJob* J) {
+static mmshift_status stats_job(const mmshift_shape* s, int64_t qfull_layer_stride, StatsJob* J,
+                                int32_t ncol = 0) {
   mmshift_status st = check_shape(s);
   if (st != MMSHIFT_OK) return st;
   std::memset(J, 0, sizeof(*J));
   J->L = s->n_layers;
   J->B = s->batch;
-  J->ncol = s->n_q_heads * s->head_dim;
+  J->ncol = ncol ? ncol : s->n_q_heads * s->head_dim;
+  if (J->ncol % 8) return MMSHIFT_ERR_INVALID_ARG;
   const int64_t total = s->cu_seqlens[s->batch];
   int maxc = 0;
   for (int b = 0; b < s->batch; ++b) {
@@ -253,6 +255,38 @@ static mmshift_status stats_job(const mmshift_shape* s, int64_t qfull_layer_stri
   J->ls = qfull_layer_stride ? qfull_layer_stride : dense;
   if (J->L > 1 && J->ls < dense) return MMSHIFT_ERR_INVALID_ARG;
   if (J->ls % 8) return MMSHIFT_ERR_INVALID_ARG;   // 16-byte rows for the vector loads
+  return MMSHIFT_OK;
+}
+
+// The hidden-space proxy job of a call: shapes, tiles and RoPE positions.
+static mmshift_status hidden_job(const mmshift_shape* s, int32_t d_model, const mmshift_params* p,
+                                 const int32_t* rope_pos, HiddenJob* J) {
+  mmshift_status st = check_shape(s);
+  if (st != MMSHIFT_OK) return st;
+  if ((st = check_params(p)) != MMSHIFT_OK) return st;
+  if (s->dtype != MMSHIFT_BF16) return MMSHIFT_ERR_UNSUPPORTED;
+  if (d_model < 64 || d_model % 64) return MMSHIFT_ERR_UNSUPPORTED;
+  const int F = s->n_q_heads * s->head_dim;
+  if (F % 128) return MMSHIFT_ERR_UNSUPPORTED;
+  std::memset(J, 0, sizeof(*J));
+  J->L = s->n_layers;
+  J->B = s->batch;
+  J->Hq = s->n_q_heads;
+  J->d = s->head_dim;
+  J->F = F;
+  J->DM = d_model;
+  J->N = p->n_proxies;
+  J->Npad = (p->n_proxies + 127) / 128 * 128;
+  J->NT = F % 256 == 0 ? 256 : 128;
+  J->MT = J->Npad / 128;
+  J->NTL = F / J->NT;
+  J->tiles = J->L * J->B * J->MT * J->NTL;
+  J->gamma = p->gamma;
+  J->rope_theta = p->rope_theta;
+  J->seed = p->seed;
+  J->layer_id0 = p->layer_id;
+  for (int b = 0; b < s->batch; ++b)
+    J->pos[b] = rope_pos ? rope_pos[b] : (s->cu_seqlens[b + 1] - s->cu_seqlens[b]) + p->rope_pos_offset;
   return MMSHIFT_OK;
 }
 
@@ -359,6 +393,71 @@ mmshift_status mmshift_prefill_stats(const mmshift_shape* s, const void* Qfull,
   if (workspace_bytes < need) return MMSHIFT_ERR_WORKSPACE;
   const cudaError_t e = launch_prefill_stats(J, Qfull, static_cast<float*>(workspace), stats,
                                              (cudaStream_t)stream, s->dtype == MMSHIFT_BF16);
+  return e == cudaSuccess ? MMSHIFT_OK : cuda_fail(e);
+}
+
+mmshift_status mmshift_hidden_stats_workspace_size(const mmshift_shape* s, int32_t d_model,
+                                                  size_t* bytes) {
+  if (!bytes || d_model < 8) return MMSHIFT_ERR_INVALID_ARG;
+  StatsJob J;
+  const mmshift_status st = stats_job(s, 0, &J, d_model);
+  if (st != MMSHIFT_OK) return st;
+  *bytes = align256((size_t)J.L * J.B * J.nchunk * 3 * J.ncol * sizeof(float));
+  return MMSHIFT_OK;
+}
+
+mmshift_status mmshift_hidden_stats(const mmshift_shape* s, int32_t d_model, const void* H,
+                                    int64_t h_layer_stride, float* stats, void* workspace,
+                                    size_t workspace_bytes, mmshift_stream_t stream) {
+  if (d_model < 8) return MMSHIFT_ERR_INVALID_ARG;
+  StatsJob J;
+  mmshift_status st = stats_job(s, h_layer_stride, &J, d_model);
+  if (st != MMSHIFT_OK) return st;
+  if (!H || !stats || !workspace) return MMSHIFT_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(H) & 15) return MMSHIFT_ERR_INVALID_ARG;
+  size_t need = 0;
+  if ((st = mmshift_hidden_stats_workspace_size(s, d_model, &need)) != MMSHIFT_OK) return st;
+  if (workspace_bytes < need) return MMSHIFT_ERR_WORKSPACE;
+  const cudaError_t e = launch_prefill_stats(J, H, static_cast<float*>(workspace), stats,
+                                             (cudaStream_t)stream, s->dtype == MMSHIFT_BF16);
+  return e == cudaSuccess ? MMSHIFT_OK : cuda_fail(e);
+}
+
+mmshift_status mmshift_hidden_proxies_workspace_size(const mmshift_shape* s, int32_t d_model,
+                                                     const mmshift_params* p, size_t* bytes) {
+  if (!bytes) return MMSHIFT_ERR_INVALID_ARG;
+  HiddenJob J;
+  const mmshift_status st = hidden_job(s, d_model, p, nullptr, &J);
+  if (st != MMSHIFT_OK) return st;
+  *bytes = 256 + hidden_scratch_bytes(J);
+  return MMSHIFT_OK;
+}
+
+mmshift_status mmshift_build_hidden_proxies(const mmshift_shape* s, int32_t d_model,
+                                            const float* hstats, const void* W_Q,
+                                            int64_t wq_layer_stride, const void* bias_q,
+                                            const int32_t* rope_pos, const mmshift_params* p,
+                                            void* proxies, void* workspace,
+                                            size_t workspace_bytes, mmshift_stream_t stream) {
+  HiddenJob J;
+  mmshift_status st = hidden_job(s, d_model, p, rope_pos, &J);
+  if (st != MMSHIFT_OK) return st;
+  if (J.N == 0) return MMSHIFT_OK;
+  if (!hstats || !W_Q || !proxies || !workspace) return MMSHIFT_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(W_Q) & 15) || (reinterpret_cast<uintptr_t>(workspace) & 255))
+    return MMSHIFT_ERR_INVALID_ARG;
+  const int64_t dense = (int64_t)J.F * J.DM;
+  if (wq_layer_stride % 8 || (J.L > 1 && wq_layer_stride && wq_layer_stride < dense))
+    return MMSHIFT_ERR_INVALID_ARG;
+  if (J.L > 1 && wq_layer_stride == 0) wq_layer_stride = dense;
+  if (workspace_bytes < 256 + hidden_scratch_bytes(J)) return MMSHIFT_ERR_WORKSPACE;
+  if (!tmap_encoder_available()) return MMSHIFT_ERR_UNSUPPORTED;
+  J.hstats = hstats;
+  J.bias = static_cast<const __nv_bfloat16*>(bias_q);
+  J.out = static_cast<__nv_bfloat16*>(proxies);
+  J.status = static_cast<int*>(workspace);
+  const cudaError_t e = launch_hidden_proxies(J, static_cast<unsigned char*>(workspace) + 256, W_Q,
+                                              wq_layer_stride, (cudaStream_t)stream);
   return e == cudaSuccess ? MMSHIFT_OK : cuda_fail(e);
 }
 

@@ -1,6 +1,7 @@
 // Internal definitions shared by the kernels and the host entry points.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
@@ -79,6 +80,23 @@ struct StatsJob {
   int32_t tok_off[MMSHIFT_MAX_BATCH];
 };
 
+// Hidden-space proxy job (hidden.cu): per (layer, request) N proxy hidden
+// states sampled in d_model dims and projected by W_Q [F = Hq*d][d_model].
+struct HiddenJob {
+  int32_t L, B, Hq, d, F, DM, N, Npad;  // Npad = roundup(N, 128)
+  int32_t NT, MT, NTL, tiles;           // feature tile width, proxy / feature tiles, total tiles
+  float gamma, rope_theta;
+  uint64_t seed;
+  int32_t layer_id0;
+  int32_t pos[MMSHIFT_MAX_BATCH];       // RoPE position of each request's proxies
+  const float* hstats;                  // [L][B][2][DM] mean, std of the hidden states
+  const __nv_bfloat16* bias;            // [L][F] or null
+  float* rope;                          // [B][d/2][2] cos, sin (scratch) or null
+  __nv_bfloat16* hs;                    // [L][B][Npad][DM] sampled hidden states (scratch)
+  __nv_bfloat16* out;                   // [L][B][Hq][N][d] proxies
+  int* status;
+};
+
 // Row p of the packed proxy block of KV head h: which group / query head /
 // proxy it holds, or that it is padding.
 struct RowKind {
@@ -146,6 +164,17 @@ cudaError_t launch_score_simt(const Problem& P, const Buffers& bf, cudaStream_t 
 cudaError_t launch_score_umma(const Problem& P, const Buffers& bf, cudaStream_t st,
                               const void* K, cudaEvent_t* ev);
 bool umma_supported(const Problem& P);
+// Scratch of launch_hidden_proxies (sampled hidden states, RoPE table) and
+// the launch itself: sampling kernel, then the projection GEMM.
+size_t hidden_scratch_bytes(const HiddenJob& J);
+cudaError_t launch_hidden_proxies(HiddenJob J, void* scratch, const void* W, int64_t w_layer_stride,
+                                  cudaStream_t st);
+// Tiled TMA descriptor of a 3-D bf16 tensor (dims d0 innermost): boxes of
+// 64 x box1 x 1 elements, 128-byte swizzle; false if the driver's encoder is
+// unavailable or rejects the layout.
+bool make_tmap_bf16_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
+                       uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t box1);
+bool tmap_encoder_available();
 int umma_launches(const Problem& P);
 cudaError_t launch_merge(const Problem& P, const Buffers& bf, cudaStream_t st);
 cudaError_t launch_cover(const Problem& P, const Buffers& bf, cudaStream_t st);

@@ -680,33 +680,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
 }
 
 // ---------------------------------------------------------------- host side
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-  static std::once_flag once;
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  std::call_once(once, [] {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
-                                         &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  });
-  return fn;
-}
-
-bool make_map_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
-                 uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t box1) {
-  auto fn = encode_fn();
-  if (!fn) return false;
-  const cuuint64_t dims[3] = {d0, d1, d2};
-  const cuuint64_t strides[2] = {stride1_bytes, stride2_bytes};
-  const cuuint32_t box[3] = {64, box1, 1};
-  const cuuint32_t es[3] = {1, 1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 Sched make_sched(const Problem& P, int pass) {
   Sched s;
   memset(&s, 0, sizeof(s));
@@ -742,10 +715,10 @@ cudaError_t launch_d(const Problem& P, const Buffers& bf, cudaStream_t st, const
   using SM = Smem<D>;
   CUtensorMap kmap, pmap;
   const uint64_t ls = P.L > 1 ? (uint64_t)P.ls_kv : (uint64_t)P.total_T * P.Hkv * D;
-  if (!make_map_3d(&kmap, K, (uint64_t)P.Hkv * D, (uint64_t)P.total_T, (uint64_t)P.L,
+  if (!make_tmap_bf16_3d(&kmap, K, (uint64_t)P.Hkv * D, (uint64_t)P.total_T, (uint64_t)P.L,
                    (uint64_t)P.Hkv * D * 2, ls * 2, BK))
     return cudaErrorInvalidValue;
-  if (!make_map_3d(&pmap, bf.packed, D, (uint64_t)P.Prows_pad, (uint64_t)P.L * P.B * P.Hkv,
+  if (!make_tmap_bf16_3d(&pmap, bf.packed, D, (uint64_t)P.Prows_pad, (uint64_t)P.L * P.B * P.Hkv,
                    (uint64_t)D * 2, (uint64_t)P.Prows_pad * D * 2, 16))
     return cudaErrorInvalidValue;
   const int nsm = sm_count();
@@ -785,6 +758,35 @@ cudaError_t launch_d(const Problem& P, const Buffers& bf, cudaStream_t st, const
 
 }  // namespace
 
+static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static std::once_flag once;
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+bool make_tmap_bf16_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
+                       uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t box1) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[3] = {d0, d1, d2};
+  const cuuint64_t strides[2] = {stride1_bytes, stride2_bytes};
+  const cuuint32_t box[3] = {64, box1, 1};
+  const cuuint32_t es[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool tmap_encoder_available() { return encode_fn() != nullptr; }
+
 bool umma_supported(const Problem& P) {
   if (P.dtype != MMSHIFT_BF16 || (P.d != 64 && P.d != 128)) return false;
   if (P.RG > SROWS || P.anchor_rows > SROWS || P.Prows_pad % SROWS) return false;
@@ -793,7 +795,7 @@ bool umma_supported(const Problem& P) {
   if (cudaGetDevice(&dev) != cudaSuccess) return false;
   if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess)
     return false;
-  return major == 10 && encode_fn() != nullptr;
+  return major == 10 && tmap_encoder_available();
 }
 
 int umma_launches(const Problem& P) { (void)P; return 3; }

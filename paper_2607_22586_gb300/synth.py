@@ -243,6 +243,40 @@ def make_prompt_queries(wl: Workload, layer: int, li: LayerInputs,
     return out
 
 
+def make_hidden_states(wl: Workload, layer: int, d_model: int,
+                       seed_tag: int = 0x48494444) -> np.ndarray:
+    """Prefill hidden states of one layer, [total_T, d_model] (dtype-exact
+    float32): per feature a mean N(0, 0.5^2) and a scale U(0.5, 1.5) shared by
+    the requests, four massive-activation features with mean +-20 (large,
+    nearly constant features of LLM residual streams), a per-request
+    N(0, 0.5^2) modality offset on visual positions, unit normal noise."""
+    rng = np.random.Generator(np.random.Philox(key=[wl.seed ^ seed_tag, layer]))
+    mean = rng.normal(0.0, 0.5, size=d_model).astype(np.float32)
+    scale = rng.uniform(0.5, 1.5, size=d_model).astype(np.float32)
+    massive = rng.choice(d_model, size=min(4, d_model), replace=False)
+    mean[massive] = np.float32(20.0) * np.sign(rng.standard_normal(massive.size)).astype(np.float32)
+    out = np.empty((wl.total_tokens, d_model), dtype=np.float32)
+    cu = wl.cu_seqlens()
+    for b, (t_len, n_vis) in enumerate(zip(wl.seq_lens, wl.n_visual)):
+        h = mean[None, :] + scale[None, :] * rng.standard_normal((t_len, d_model), dtype=np.float32)
+        h[:n_vis] += np.float32(0.5) * rng.standard_normal(d_model, dtype=np.float32)[None]
+        out[cu[b]:cu[b + 1]] = round_to_dtype(h, wl.dtype)
+    return out
+
+
+def make_query_projection(wl: Workload, layer: int, d_model: int, with_bias: bool = True,
+                          seed_tag: int = 0x57515052):
+    """Query projection of one layer: W_Q [Hq*d, d_model] with entries
+    N(0, 1/d_model) (so projected proxies have O(1) features) and a bias
+    [Hq*d] N(0, 0.5^2) or None; dtype-exact float32."""
+    rng = np.random.Generator(np.random.Philox(key=[wl.seed ^ seed_tag, layer]))
+    f = wl.n_q_heads * wl.head_dim
+    w = rng.standard_normal((f, d_model), dtype=np.float32) * np.float32(1.0 / np.sqrt(d_model))
+    bias = (rng.standard_normal(f, dtype=np.float32) * np.float32(0.5)) if with_bias else None
+    return (round_to_dtype(w, wl.dtype),
+            None if bias is None else round_to_dtype(bias, wl.dtype))
+
+
 def make_proxies(wl: Workload, n_proxies: int, layer: int, scale: float = 8.0,
                  seed_tag: int = 0x50524F58) -> np.ndarray:
     """Seeded stand-alone proxy set [B, Hq, N_p, d] (dtype-exact float32).

@@ -110,3 +110,42 @@ def test_prefill_stats_validation_before_any_launch():
     p = M.default_params()
     assert M.mmshift_build_proxies_from_stats(s, None, p, fake) == L.MMSHIFT_ERR_INVALID_ARG
     assert M.mmshift_build_proxies_from_stats(s, fake, p, None) == L.MMSHIFT_ERR_INVALID_ARG
+
+
+def test_hidden_entries_validation_before_any_launch():
+    s = _shape()
+    p = M.default_params()
+    dm = 1024
+    n = M.mmshift_hidden_stats_workspace_size(s, dm)
+    assert n == ((1 * 2 * 1 * 3 * dm * 4 + 255) // 256) * 256
+    fake = 1 << 40
+    assert M.mmshift_hidden_stats(s, dm, None, 0, fake, fake, n) == L.MMSHIFT_ERR_INVALID_ARG
+    assert M.mmshift_hidden_stats(s, dm, fake + 8, 0, fake, fake, n) == L.MMSHIFT_ERR_INVALID_ARG
+    assert M.mmshift_hidden_stats(s, dm, fake, 0, fake, fake, n - 256) == L.MMSHIFT_ERR_WORKSPACE
+    assert M.mmshift_hidden_stats(s, 1020, fake, 0, fake, fake, n) == L.MMSHIFT_ERR_INVALID_ARG
+    # hidden proxies: N = 512 proxies -> 4 tiles of 128 rows, sampled states in the workspace
+    w = M.mmshift_hidden_proxies_workspace_size(s, dm, p)
+    assert w >= 256 + 2 * 512 * dm * 2
+    args = dict(hstats=fake, W_Q=fake, wq_layer_stride=0, bias_q=None, rope_pos=None, params=p,
+                proxies=fake, workspace=fake, workspace_bytes=w)
+
+    def call(shape=s, d_model=dm, **kw):
+        a = dict(args)
+        a.update(kw)
+        return M.mmshift_build_hidden_proxies(shape, d_model, a["hstats"], a["W_Q"], a["wq_layer_stride"],
+                                              a["bias_q"], a["rope_pos"], a["params"], a["proxies"],
+                                              a["workspace"], a["workspace_bytes"])
+
+    assert call(W_Q=None) == L.MMSHIFT_ERR_INVALID_ARG
+    assert call(hstats=None) == L.MMSHIFT_ERR_INVALID_ARG
+    assert call(W_Q=fake + 4) == L.MMSHIFT_ERR_INVALID_ARG            # unaligned weights
+    assert call(workspace=fake + 16) == L.MMSHIFT_ERR_INVALID_ARG      # unaligned workspace
+    assert call(wq_layer_stride=12) == L.MMSHIFT_ERR_INVALID_ARG       # stride not a multiple of 8
+    assert call(workspace_bytes=w - 256) == L.MMSHIFT_ERR_WORKSPACE
+    assert call(d_model=1000) == L.MMSHIFT_ERR_UNSUPPORTED             # not a multiple of 64
+    assert call(shape=_shape(dtype=1)) == L.MMSHIFT_ERR_UNSUPPORTED     # bf16 only
+    assert call(shape=_shape(n_q_heads=3, n_kv_heads=1, head_dim=64)) == L.MMSHIFT_ERR_UNSUPPORTED
+    s2 = _shape(n_layers=2, layer_stride_kv=250 * 2 * 128, layer_stride_q=2 * 8 * 8 * 128)
+    w2 = M.mmshift_hidden_proxies_workspace_size(s2, dm, p)
+    assert call(shape=s2, wq_layer_stride=8 * 128 * dm - 8, workspace_bytes=w2) == L.MMSHIFT_ERR_INVALID_ARG
+    assert call(params=M.default_params(n_proxies=0, n_groups=0)) == L.MMSHIFT_OK   # nothing to do
