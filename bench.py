@@ -17,6 +17,12 @@ step's algorithmic bytes (K read once + K/V gathered, read and written) reach.
 of the window's (Section 3.2.1): each step then also reads the L x T x Hq x d
 prompt queries once (mmshift_prefill_stats) and selects with
 mmshift_select_with_stats; the line adds that pass's HBM roofline.
+--stats hidden builds the proxies the paper's way: statistics over the prefill
+hidden states (d_model = Hq x d = 3584 features per token, 6.6 GB per step),
+N proxy hidden states projected by a resident W_Q on the tensor cores
+(mmshift_hidden_stats + mmshift_build_hidden_proxies), then mmshift_select
+with those proxies; the line adds the statistics pass's HBM roofline and the
+projection's tensor roofline.
 
 --impl reference times the CPU oracle on the host cores instead (a bounded
 sample of the same workload per step).
@@ -109,6 +115,99 @@ def prompt_queries_device(wl, K, Qwin, seed: int):
             nw = min(w, t_len)
             out[l, hi - nw:hi] = Qv[l, b, w - nw:]
     return out.view(L, -1)
+
+
+def hidden_states_device(wl, d_model: int, seed: int, device):
+    """Prefill hidden states [L, T*d_model] on the device for --stats hidden,
+    with the recipe of synth.make_hidden_states (per-feature mean N(0, 0.5^2)
+    with four massive features at +-20, scale U(0.5, 1.5), a 0.5 N(0, 1)
+    modality offset on visual positions, unit noise), drawn by torch's seeded
+    device generator."""
+    import torch
+    L, T = wl.n_layers, wl.total_tokens
+    g = torch.Generator(device=device).manual_seed(seed)
+    out = torch.empty((L, T, d_model), dtype=torch.bfloat16, device=device)
+    cu = wl.cu_seqlens()
+    for l in range(L):
+        mean = torch.randn(d_model, generator=g, device=device) * 0.5
+        scale = torch.rand(d_model, generator=g, device=device) + 0.5
+        massive = torch.randperm(d_model, generator=g, device=device)[:4]
+        mean[massive] = 20.0 * torch.sign(torch.randn(4, generator=g, device=device))
+        for b, (t_len, n_vis) in enumerate(zip(wl.seq_lens, wl.n_visual)):
+            h = mean + scale * torch.randn((t_len, d_model), generator=g, device=device)
+            h[:n_vis] += 0.5 * torch.randn(d_model, generator=g, device=device)
+            out[l, int(cu[b]):int(cu[b + 1])] = h.to(torch.bfloat16)
+    return out.view(L, -1)
+
+
+def query_projection_device(wl, d_model: int, seed: int, device):
+    """W_Q [L, Hq*d, d_model] with N(0, 1/d_model) entries and a bias
+    [L, Hq*d] N(0, 0.5^2), bf16, as synth.make_query_projection: model weights,
+    resident on the device (not per-step inputs)."""
+    import torch
+    f = wl.n_q_heads * wl.head_dim
+    g = torch.Generator(device=device).manual_seed(seed)
+    w = (torch.randn((wl.n_layers, f, d_model), generator=g, device=device) / math.sqrt(d_model))
+    bias = torch.randn((wl.n_layers, f), generator=g, device=device) * 0.5
+    return w.to(torch.bfloat16), bias.to(torch.bfloat16)
+
+
+class PreStep:
+    """What runs before the selection when the proxies' statistics do not come
+    from the window: --stats prefill (statistics over every prompt query, then
+    mmshift_select_with_stats) or --stats hidden (statistics over the prefill
+    hidden states, hidden-space proxies projected by W_Q, then mmshift_select
+    with them). ``x`` is the per-step input (prompt queries or hidden states)."""
+
+    def __init__(self, kind, wl, shape, params, K, Q, seed, d_model, M):
+        import torch
+        self.kind, self.wl, self.shape, self.params, self.M = kind, wl, shape, params, M
+        dev = K.device
+        L, B = wl.n_layers, wl.batch
+        if kind == "prefill":
+            self.x = prompt_queries_device(wl, K, Q, seed=seed)
+            self.ncol = wl.n_q_heads * wl.head_dim
+            self.ws_bytes = M.mmshift_prefill_stats_workspace_size(shape)
+            self.stages = ["prefill_stats"]
+            self.launches = 2
+        else:
+            self.dm = d_model
+            self.x = hidden_states_device(wl, d_model, seed, dev)
+            self.W, self.bias = query_projection_device(wl, d_model, seed + 1, dev)
+            self.ncol = d_model
+            self.ws_bytes = M.mmshift_hidden_stats_workspace_size(shape, d_model)
+            self.hp_bytes = M.mmshift_hidden_proxies_workspace_size(shape, d_model, params)
+            self.hws = torch.zeros(self.hp_bytes, dtype=torch.uint8, device=dev)
+            self.px = torch.empty((L, B, wl.n_q_heads, params.n_proxies, wl.head_dim),
+                                  dtype=torch.bfloat16, device=dev)
+            self.stages = ["hidden_stats", "hidden_proxies"]
+            self.launches = 4
+        self.ws = torch.zeros(self.ws_bytes, dtype=torch.uint8, device=dev)
+        self.stats = torch.empty((L, B, 2, self.ncol), device=dev)
+
+    def run(self, x, stream, sev=None):
+        """Launch the pre-selection steps on ``stream``; sev (nullable) gets
+        an event before and after each. Returns the statistics (prefill) or
+        the proxies (hidden) the selection takes."""
+        M = self.M
+        if sev:
+            sev[0].record(stream)
+        if self.kind == "prefill":
+            M.check(M.mmshift_prefill_stats(self.shape, x, 0, self.stats, self.ws, self.ws_bytes,
+                                            stream), "mmshift_prefill_stats")
+            if sev:
+                sev[1].record(stream)
+            return self.stats
+        M.check(M.mmshift_hidden_stats(self.shape, self.dm, x, 0, self.stats, self.ws, self.ws_bytes,
+                                       stream), "mmshift_hidden_stats")
+        if sev:
+            sev[1].record(stream)
+        M.check(M.mmshift_build_hidden_proxies(self.shape, self.dm, self.stats, self.W, 0, self.bias,
+                                               None, self.params, self.px, self.hws, self.hp_bytes,
+                                               stream), "mmshift_build_hidden_proxies")
+        if sev:
+            sev[2].record(stream)
+        return self.px
 
 
 def read_peaks():
@@ -372,29 +471,26 @@ def run_gpu(args, wl):
     out_v = torch.empty_like(out_k)
     stream = torch.cuda.current_stream(dev)
     nst = LB.MMSHIFT_N_STAGES + 1
-    prefill = args.stats == "prefill"
-    if prefill:
-        Qf = prompt_queries_device(wl, K, Q, seed=wl.seed + 7919 * (rank + 1))
-        st_bytes = M.mmshift_prefill_stats_workspace_size(shape)
-        st_ws = torch.zeros(st_bytes, dtype=torch.uint8, device=dev)
-        stats = torch.empty((L, wl.batch, 2, wl.n_q_heads * wl.head_dim), device=dev)
+    d_model = args.d_model or wl.n_q_heads * wl.head_dim
+    pre = None
+    if args.stats != "window":
+        pre = PreStep(args.stats, wl, shape, params, K, Q, wl.seed + 7919 * (rank + 1), d_model, M)
 
-    def select(Kx, Vx, Qx, Qfx, dbg=None, sev=None):
-        if not prefill:
+    def select(Kx, Vx, Qx, Xx, dbg=None, sev=None):
+        if pre is None:
             M.check(M.mmshift_select(shape, Kx, Vx, Qx, None, params, out_idx, out_k, out_v, dbg,
                                      ws, ws_bytes, stream), "mmshift_select")
-            return
-        if sev:
-            sev[0].record(stream)
-        M.check(M.mmshift_prefill_stats(shape, Qfx, 0, stats, st_ws, st_bytes, stream),
-                "mmshift_prefill_stats")
-        if sev:
-            sev[1].record(stream)
-        M.check(M.mmshift_select_with_stats(shape, Kx, Vx, Qx, stats, params, out_idx, out_k, out_v,
-                                            dbg, ws, ws_bytes, stream), "mmshift_select_with_stats")
+        elif pre.kind == "prefill":
+            st = pre.run(Xx, stream, sev)
+            M.check(M.mmshift_select_with_stats(shape, Kx, Vx, Qx, st, params, out_idx, out_k, out_v,
+                                                dbg, ws, ws_bytes, stream), "mmshift_select_with_stats")
+        else:
+            px = pre.run(Xx, stream, sev)
+            M.check(M.mmshift_select(shape, Kx, Vx, Qx, px, params, out_idx, out_k, out_v, dbg,
+                                     ws, ws_bytes, stream), "mmshift_select")
 
     def step(dbg=None, sev=None):
-        select(K, V, Q, Qf if prefill else None, dbg, sev)
+        select(K, V, Q, pre.x if pre else None, dbg, sev)
 
     for _ in range(args.warmup):
         step()
@@ -406,7 +502,7 @@ def run_gpu(args, wl):
         for ev in evs:
             ev.record(stream)
     dbgs = [M.make_debug(stage_events=ev) for ev in stage_ev]
-    stat_ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] if prefill else None
+    stat_ev = [[torch.cuda.Event(enable_timing=True) for _ in range(len(pre.stages) + 1)] if pre else None
                for _ in range(args.steps)]
     clocks = ClockSampler(torch.cuda.current_device())
     clocks.start()
@@ -426,10 +522,10 @@ def run_gpu(args, wl):
     stage_ms = {name: statistics.mean(ev[i].elapsed_time(ev[i + 1]) for ev in stage_ev)
                 for i, name in enumerate(LB.STAGES)}
     launches = dbgs[0].launches * args.steps
-    if prefill:
-        stage_ms = {"prefill_stats": statistics.mean(e[0].elapsed_time(e[1]) for e in stat_ev),
-                    **stage_ms}
-        launches += 2 * args.steps        # partial sums + merge
+    if pre:
+        stage_ms = {**{name: statistics.mean(e[i].elapsed_time(e[i + 1]) for e in stat_ev)
+                       for i, name in enumerate(pre.stages)}, **stage_ms}
+        launches += pre.launches * args.steps
 
     # end to end through the same C ABI call: host buffers in, results out
     idx_h = torch.empty(out_idx.shape, dtype=out_idx.dtype, pin_memory=True)
@@ -441,10 +537,10 @@ def run_gpu(args, wl):
     # copies of step k+1 (on a copy stream) overlap the selection of step k;
     # a buffer is refilled only after the selection that read it.
     Kb, Vb, Qb = [K, torch.empty_like(K)], [V, torch.empty_like(V)], [Q, torch.empty_like(Q)]
-    if prefill:
-        Qf_pin = torch.empty(Qf.shape, dtype=Qf.dtype, pin_memory=True)
-        Qf_pin.copy_(Qf)
-        Qfb = [Qf, torch.empty_like(Qf)]
+    if pre:
+        X_pin = torch.empty(pre.x.shape, dtype=pre.x.dtype, pin_memory=True)
+        X_pin.copy_(pre.x)
+        Xb = [pre.x, torch.empty_like(pre.x)]
     cstream = torch.cuda.Stream(dev)
     ready = [torch.cuda.Event() for _ in range(2)]
     free = [torch.cuda.Event() for _ in range(2)]
@@ -455,13 +551,13 @@ def run_gpu(args, wl):
             Kb[i].copy_(K_pin, non_blocking=True)
             Vb[i].copy_(V_pin, non_blocking=True)
             Qb[i].copy_(Q_pin, non_blocking=True)
-            if prefill:
-                Qfb[i].copy_(Qf_pin, non_blocking=True)
+            if pre:
+                Xb[i].copy_(X_pin, non_blocking=True)
         ready[i].record(cstream)
 
     def select_out(i):
         stream.wait_event(ready[i])
-        select(Kb[i], Vb[i], Qb[i], Qfb[i] if prefill else None)
+        select(Kb[i], Vb[i], Qb[i], Xb[i] if pre else None)
         free[i].record(stream)
         idx_h.copy_(out_idx, non_blocking=True)
         ok_h.copy_(out_k, non_blocking=True)
@@ -486,24 +582,38 @@ def run_gpu(args, wl):
     torch.cuda.synchronize()
     e_ms = ranks.max(e0.elapsed_time(e1) / e_steps, dev)
     h2d = sum(t.numel() * t.element_size() for t in (K_pin, V_pin, Q_pin))
-    if prefill:
-        h2d += Qf_pin.numel() * Qf_pin.element_size()
+    if pre:
+        h2d += X_pin.numel() * X_pin.element_size()
     d2h = sum(t.numel() * t.element_size() for t in (idx_h, ok_h, ov_h))
 
     bytes_step, k_read, pass_flops = algorithmic(wl, hyper)
-    stats_roof = None
-    if prefill:
-        # algorithmic bytes of the statistics pass: every prompt query read
-        # once, the [L, B, 2, Hq*d] float32 statistics written
-        q_bytes = Qf.numel() * Qf.element_size()
-        s_bytes = q_bytes + stats.numel() * 4
-        bytes_step += q_bytes
-        st_ms = stage_ms["prefill_stats"]
+    extra_roofs = {}
+    if pre:
+        # algorithmic bytes of the statistics pass: every prompt query (or
+        # hidden state) read once, the [L, B, 2, ncol] float32 statistics written
+        x_bytes = pre.x.numel() * pre.x.element_size()
+        s_bytes = x_bytes + pre.stats.numel() * 4
+        bytes_step += x_bytes
+        st_ms = stage_ms[pre.stages[0]]
         ach = s_bytes / (st_ms * 1e-3) / 1e9
-        stats_roof = {"bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                      "frac": ach / peaks["hbm_gbs"], "traffic": stats_traffic(wl),
-                      "kernel": "stats_partial_kernel + stats_merge_kernel",
-                      "bytes_per_launch": s_bytes, "peak_kind": f"HBM copy ({peak_src})"}
+        extra_roofs[pre.stages[0] + "_roofline"] = {
+            "bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+            "frac": ach / peaks["hbm_gbs"],
+            "traffic": stats_traffic(wl) if pre.kind == "prefill" else None,
+            "kernel": "stats_partial_kernel + stats_merge_kernel",
+            "bytes_per_launch": s_bytes, "peak_kind": f"HBM copy ({peak_src})"}
+        if pre.kind == "hidden":
+            # the projection: 2 * N * d_model * Hq*d flops per (layer, request);
+            # the stage also holds the sampling kernel
+            f_ms = stage_ms["hidden_proxies"]
+            flops = 2.0 * hyper["n_proxies"] * d_model * wl.n_q_heads * wl.head_dim * L * wl.batch
+            tpeak = float(peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]))
+            ach = flops / (f_ms * 1e-3) / 1e12
+            extra_roofs["hidden_proxies_roofline"] = {
+                "bound": "tensor", "achieved": ach, "peak": tpeak, "unit": "TFLOP/s",
+                "frac": ach / tpeak, "traffic": None,
+                "kernel": "hidden_sample_kernel + hidden_proj_kernel",
+                "flops_per_launch": flops, "peak_kind": f"bf16 dense, sustained ({peak_src})"}
     tokens_layer = T * L * world          # metric unit: tokens per second per layer
     value = job_value(T * L, world, ms)
     hbm_frac = bytes_step / (ms * 1e-3) / (peaks["hbm_gbs"] * 1e9)
@@ -551,13 +661,14 @@ def run_gpu(args, wl):
                    "n_proxies": hyper["n_proxies"], "n_groups": hyper["n_groups"],
                    "gamma": hyper["gamma"], "tau": hyper["tau"], "lambda": hyper["lam"],
                    "stats": args.stats,
+                   **({"d_model": d_model} if args.stats == "hidden" else {}),
                    "l2": "inputs (K+V %.2f GB) larger than L2; no flush" % (2 * k_read / 1e9),
                    "parallelism": f"replicas x{world}"},
         "hbm_roofline_frac": hbm_frac,
         "hbm_bytes_per_step": bytes_step,
         "stage_ms": stage_ms,
         "roofline": roof,
-        **({"prefill_stats_roofline": stats_roof} if stats_roof else {}),
+        **extra_roofs,
         "cpu_baseline": cpu,
         "e2e": {"value": job_value(T * L, world, e_ms), "unit": UNIT, "ms_per_step": e_ms,
                 "pipeline": "inputs double-buffered on the device: the host-to-device copies "
@@ -584,9 +695,13 @@ def main(argv=None):
                     help="use only the first N layers of the workload (profiling runs)")
     ap.add_argument("--proxies", choices=["paper", "few"], default="paper",
                     help="paper: N=512, G=32 (Section 4.1); few: N=W, G=W/16")
-    ap.add_argument("--stats", choices=["window", "prefill"], default="window",
-                    help="proxy statistics: over the W window queries, or over every prompt "
-                         "query (mmshift_prefill_stats + mmshift_select_with_stats)")
+    ap.add_argument("--stats", choices=["window", "prefill", "hidden"], default="window",
+                    help="proxy statistics: over the W window queries; over every prompt query "
+                         "(mmshift_prefill_stats + mmshift_select_with_stats); or over the prefill "
+                         "hidden states with proxies projected by W_Q (mmshift_hidden_stats + "
+                         "mmshift_build_hidden_proxies + mmshift_select)")
+    ap.add_argument("--d-model", type=int, default=0,
+                    help="hidden size for --stats hidden (0: Hq * d, as in Qwen2.5-VL-7B)")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="CPU oracle sample budget for cpu_baseline (0 disables)")
     ap.add_argument("--ref-seconds", type=float, default=8.0,
