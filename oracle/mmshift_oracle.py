@@ -34,7 +34,7 @@ __all__ = [
     "proxy_normals", "window_stats", "prefill_stats", "rope_rotate", "round_to",
     "build_proxies", "build_proxies_from_stats", "hidden_normals", "hidden_proxies",
     "softmax_rows", "group_masses", "anchor_attention", "cover_sets", "votes",
-    "scores", "select_topk", "gather", "select_request", "select",
+    "scores", "select_topk", "gather", "attention_coverage", "select_request", "select",
 ]
 
 # ---------------------------------------------------------------------------
@@ -379,6 +379,33 @@ def gather(keys: np.ndarray, values: np.ndarray, idx: np.ndarray):
     keys/values: [T, Hkv, d]; idx: [C', Hkv] -> two [C', Hkv, d] arrays."""
     h = np.arange(idx.shape[1])[None, :]
     return keys[idx, h], values[idx, h]
+
+
+# ---------------------------------------------------------------------------
+# Quality metric: attention-mass coverage of the kept set (§1, Fig. 1b)
+# ---------------------------------------------------------------------------
+def attention_coverage(keys: np.ndarray, dec_queries: np.ndarray, idx: np.ndarray,
+                       scale: float) -> np.ndarray:
+    """Fraction of decode-time attention probability that lands on the kept
+    prompt entries (§1, Fig. 1b's attention mass coverage).
+
+    Reading: for decode query q of query head hq, the softmax of
+    scale * q.k_t over the T prompt keys of KV head h = hq // r (the prompt
+    part of the decode-time attention, renormalised over the prompt), summed
+    over the kept indices idx[:, h].
+    keys: [T, Hkv, d]; dec_queries: [n, Hq, d]; idx: [C', Hkv] -> [Hq, n].
+    """
+    keys = np.asarray(keys, dtype=np.float64)
+    dq = np.asarray(dec_queries, dtype=np.float64)
+    t_len, hkv, _ = keys.shape
+    n, hq, _ = dq.shape
+    r = hq // hkv
+    out = np.zeros((hq, n))
+    for q in range(hq):
+        h = q // r
+        p = softmax_rows(scale * (dq[:, q, :] @ keys[:, h, :].T))     # [n, T]
+        out[q] = p[:, np.asarray(idx)[:, h]].sum(axis=1)
+    return out
 
 
 # ---------------------------------------------------------------------------

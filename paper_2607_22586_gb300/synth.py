@@ -277,6 +277,24 @@ def make_query_projection(wl: Workload, layer: int, d_model: int, with_bias: boo
             None if bias is None else round_to_dtype(bias, wl.dtype))
 
 
+def make_decode_queries(wl: Workload, layer: int, li: LayerInputs, n_dec: int,
+                        spread: float = 1.5, seed_tag: int = 0x44454351) -> np.ndarray:
+    """Synthetic decode-time queries of one layer, [B, n_dec, Hq, d]
+    (dtype-exact float32): the window recipe (half the request's per-head
+    key mean) with noise of std ``spread`` > 1, since decode-time queries
+    spread wider than prefill ones (§1, Fig. 1a)."""
+    rng = np.random.Generator(np.random.Philox(key=[wl.seed ^ seed_tag, layer]))
+    hq, hkv, d = wl.n_q_heads, wl.n_kv_heads, wl.head_dim
+    cu = wl.cu_seqlens()
+    out = np.empty((wl.batch, n_dec, hq, d), dtype=np.float32)
+    for b in range(wl.batch):
+        kmean = li.K[cu[b]:cu[b + 1]].mean(axis=0, dtype=np.float64).astype(np.float32)
+        q = (np.float32(0.5) * np.repeat(kmean, hq // hkv, axis=0)[None]
+             + np.float32(spread) * rng.standard_normal((n_dec, hq, d), dtype=np.float32))
+        out[b] = round_to_dtype(q, wl.dtype)
+    return out
+
+
 def make_proxies(wl: Workload, n_proxies: int, layer: int, scale: float = 8.0,
                  seed_tag: int = 0x50524F58) -> np.ndarray:
     """Seeded stand-alone proxy set [B, Hq, N_p, d] (dtype-exact float32).

@@ -157,6 +157,43 @@ def _hidden_normals_query_stream(seed, layer_id, b, n_proxies, d_model):
     return O.proxy_normals(seed, layer_id, b, 1, n_proxies, d_model)[0]
 
 
+def _coverage_modulo_heads(keys, dec_queries, idx, scale):
+    keys = np.asarray(keys, dtype=np.float64)
+    dq = np.asarray(dec_queries, dtype=np.float64)
+    hkv, hq = keys.shape[1], dq.shape[1]
+    out = np.zeros((hq, dq.shape[0]))
+    for q in range(hq):
+        h = q % hkv
+        p = O.softmax_rows(scale * (dq[:, q, :] @ keys[:, h, :].T))
+        out[q] = p[:, idx[:, h]].sum(axis=1)
+    return out
+
+
+def _coverage_no_scale(keys, dec_queries, idx, scale):
+    keys = np.asarray(keys, dtype=np.float64)
+    dq = np.asarray(dec_queries, dtype=np.float64)
+    hkv, hq = keys.shape[1], dq.shape[1]
+    r = hq // hkv
+    out = np.zeros((hq, dq.shape[0]))
+    for q in range(hq):
+        p = O.softmax_rows(dq[:, q, :] @ keys[:, q // r, :].T)
+        out[q] = p[:, idx[:, q // r]].sum(axis=1)
+    return out
+
+
+def _coverage_renormalised_on_kept(keys, dec_queries, idx, scale):
+    keys = np.asarray(keys, dtype=np.float64)
+    dq = np.asarray(dec_queries, dtype=np.float64)
+    hkv, hq = keys.shape[1], dq.shape[1]
+    r = hq // hkv
+    out = np.zeros((hq, dq.shape[0]))
+    for q in range(hq):
+        h = q // r
+        p = O.softmax_rows(scale * (dq[:, q, :] @ keys[idx[:, h], h, :].T))
+        out[q] = p.sum(axis=1)
+    return out
+
+
 MUTANTS = {
     "std_ddof0": ("window_stats", _window_stats_ddof0),
     "prefill_std_ddof0": ("prefill_stats", _prefill_stats_ddof0),
@@ -177,6 +214,9 @@ MUTANTS = {
     "hidden_projection_no_bias": ("hidden_proxies", _hidden_proxies_no_bias),
     "hidden_states_not_rounded": ("hidden_proxies", _hidden_proxies_unrounded_hidden),
     "hidden_normals_query_stream": ("hidden_normals", _hidden_normals_query_stream),
+    "coverage_modulo_heads": ("attention_coverage", _coverage_modulo_heads),
+    "coverage_no_scale": ("attention_coverage", _coverage_no_scale),
+    "coverage_renormalised_on_kept": ("attention_coverage", _coverage_renormalised_on_kept),
 }
 
 

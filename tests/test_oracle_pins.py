@@ -145,6 +145,49 @@ def pin_hidden_proxies(orc=O):
     assert math.isclose(z[0, 4 * 2], zz[0], rel_tol=1e-12)
 
 
+def pin_attention_coverage(orc=O):
+    """Fig. 1b's attention mass coverage: every key kept gives 1; a set and
+    its complement sum to 1; two keys give the logistic of their scaled logit
+    gap; a query's own top-C keys cover more than any other C-subset (brute
+    force); query heads 0-1 read KV head 0 (uniform keys: coverage C/T), heads
+    2-3 KV head 1 (one dominant key)."""
+    rng = np.random.default_rng(41)
+    t_len, hkv, hq, d = 9, 2, 4, 8
+    keys = rng.normal(size=(t_len, hkv, d))
+    dq = rng.normal(size=(5, hq, d))
+    every = np.repeat(np.arange(t_len)[:, None], hkv, axis=1)
+    assert np.allclose(orc.attention_coverage(keys, dq, every, 0.3), 1.0, rtol=0, atol=1e-12)
+    kept = np.array([[0, 1], [3, 4], [7, 8]])
+    rest = np.array([[t for t in range(t_len) if t not in kept[:, h]] for h in range(hkv)]).T
+    tot = orc.attention_coverage(keys, dq, kept, 0.3) + orc.attention_coverage(keys, dq, rest, 0.3)
+    assert np.allclose(tot, 1.0, rtol=0, atol=1e-12)
+    # two keys: coverage of key 0 = 1 / (1 + exp(-scale * (q.k0 - q.k1)))
+    k2 = rng.normal(size=(2, 1, d))
+    q2 = rng.normal(size=(3, 1, d))
+    scale = 1.0 / math.sqrt(d)
+    gap = (q2[:, 0, :] @ k2[0, 0]) - (q2[:, 0, :] @ k2[1, 0])
+    got = orc.attention_coverage(k2, q2, np.array([[0]]), scale)[0]
+    assert np.allclose(got, 1.0 / (1.0 + np.exp(-scale * gap)), rtol=1e-12)
+    # brute force: the query's own top-C keys are the best C-subset
+    q1 = dq[:1, :1, :]
+    k1 = keys[:, :1, :]
+    logits = (q1[0, 0] @ k1[:, 0, :].T) * 0.3
+    best = np.sort(np.argsort(-logits)[:3])
+    cov_best = orc.attention_coverage(k1, q1, best[:, None], 0.3)[0, 0]
+    for sub in itertools.combinations(range(t_len), 3):
+        c = orc.attention_coverage(k1, q1, np.array(sub)[:, None], 0.3)[0, 0]
+        assert c <= cov_best + 1e-12
+    # GQA: heads 0-1 -> KV head 0 (uniform), heads 2-3 -> KV head 1 (dominant key 5)
+    kk = np.zeros((t_len, hkv, d))
+    kk[:, 1, :] = rng.normal(size=(t_len, d)) * 0.01
+    qq = np.ones((2, hq, d))
+    kk[5, 1, :] = 50.0
+    sel = np.array([[0, 5], [1, 6], [2, 7]])
+    cov = orc.attention_coverage(kk, qq, sel, 1.0)
+    assert np.allclose(cov[:2], 3.0 / t_len, rtol=0, atol=1e-12)
+    assert np.all(cov[2:] > 1.0 - 1e-12)
+
+
 def pin_sampler_closed_form(orc=O):
     """Appendix A.2: for q ~ N(mu, Sigma), E[exp(q.k/sqrt d)] =
     exp(mu.k/sqrt d + k^T Sigma k / (2d)). With Sigma = diag((gamma*sigma)^2)
@@ -366,7 +409,7 @@ def pin_topk_bruteforce(orc=O):
 
 
 ALL_PINS = [pin_philox_vs_numpy, pin_normals_distribution, pin_window_stats, pin_prefill_stats,
-            pin_hidden_proxies,
+            pin_hidden_proxies, pin_attention_coverage,
             pin_sampler_closed_form, pin_rope, pin_round_bf16, pin_mass_totals,
             pin_sigma_zero_single_query, pin_shift_and_permutation, pin_budget_ge_t,
             pin_lastattn, pin_uniform_keys, pin_cover_bruteforce, pin_topk_bruteforce]
