@@ -24,6 +24,10 @@ N proxy hidden states projected by a resident W_Q on the tensor cores
 with those proxies; the line adds the statistics pass's HBM roofline and the
 projection's tensor roofline.
 
+After the timed steps the line reports the attention-mass coverage (Fig. 1b)
+of the kept set for 32 synthetic decode queries per (layer, request), next to
+that of the most recent tokens under the same budget (--coverage N; 0 skips).
+
 --impl reference times the CPU oracle on the host cores instead (a bounded
 sample of the same workload per step).
 
@@ -150,6 +154,78 @@ def query_projection_device(wl, d_model: int, seed: int, device):
     w = (torch.randn((wl.n_layers, f, d_model), generator=g, device=device) / math.sqrt(d_model))
     bias = torch.randn((wl.n_layers, f), generator=g, device=device) * 0.5
     return w.to(torch.bfloat16), bias.to(torch.bfloat16)
+
+
+def decode_queries_device(wl, K, n_dec: int, seed: int, spread: float = 1.5):
+    """Synthetic decode queries [L, B, Hq, n_dec, d] on the device with the
+    recipe of synth.make_decode_queries (half the request's per-head key mean
+    plus N(0, spread^2) noise), drawn by torch's seeded device generator."""
+    import torch
+    L, T = wl.n_layers, wl.total_tokens
+    hq, hkv, d = wl.n_q_heads, wl.n_kv_heads, wl.head_dim
+    g = torch.Generator(device=K.device).manual_seed(seed)
+    out = torch.empty((L, wl.batch, hq, n_dec, d), dtype=K.dtype, device=K.device)
+    cu = wl.cu_seqlens()
+    Kv = K.view(L, T, hkv, d)
+    for l in range(L):
+        for b in range(wl.batch):
+            kmean = Kv[l, int(cu[b]):int(cu[b + 1])].float().mean(dim=0).repeat_interleave(hq // hkv, dim=0)
+            q = 0.5 * kmean[:, None, :] + spread * torch.randn((hq, n_dec, d), generator=g, device=K.device)
+            out[l, b] = q.to(K.dtype)
+    return out
+
+
+def measure_coverage(args, wl, shape, K, Q, out_idx, stream, seed, M, tpeak):
+    """Attention-mass coverage (Fig. 1b) of the step's kept set for
+    args.coverage synthetic decode queries per (layer, request), next to the
+    coverage of the most recent min(C_b, T_b) tokens (a StreamingLLM-like
+    window without sinks), both through mmshift_coverage; plus the time of
+    one coverage call."""
+    import torch
+    n_dec = args.coverage
+    dec = decode_queries_device(wl, K, n_dec, seed)
+    nb = M.mmshift_coverage_workspace_size(shape, n_dec)
+    ws = torch.zeros(nb, dtype=torch.uint8, device=K.device)
+    L = wl.n_layers
+    cov = torch.empty((L, wl.batch, wl.n_kv_heads, n_dec), device=K.device)
+    recent = torch.empty_like(out_idx)
+    off = 0
+    for t_len, c in zip(wl.seq_lens, wl.budgets):
+        keep = min(c, t_len)
+        recent[:, off:off + keep, :] = torch.arange(t_len - keep, t_len, dtype=torch.int32,
+                                                    device=K.device)[None, :, None]
+        off += keep
+
+    def run(idx, out):
+        M.check(M.mmshift_coverage(shape, K, Q, dec, n_dec, 0.0, idx, out, ws, nb, stream),
+                "mmshift_coverage")
+
+    run(out_idx, cov)
+    cov_recent = torch.empty_like(cov)
+    run(recent, cov_recent)
+    M.check(M.mmshift_poll_status(ws, stream), "coverage status")
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(3):
+        run(out_idx, cov)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / 3
+    c = cov.flatten().double().cpu().numpy()
+    cr = cov_recent.flatten().double().cpu().numpy()
+    # two passes (softmax, mass) of 2 d flops per (decode query, query head, key)
+    flops = 2 * 2.0 * wl.head_dim * n_dec * wl.n_q_heads * wl.total_tokens * L
+    ach = flops / (ms * 1e-3) / 1e12
+    return {"n_decode_queries": n_dec, "queries": "0.5 * per-head key mean + N(0, 1.5^2), synthetic",
+            "mean": float(c.mean()), "p10": float(np.percentile(c, 10)), "min": float(c.min()),
+            "recent_window_mean": float(cr.mean()), "recent_window_p10": float(np.percentile(cr, 10)),
+            "ms_per_call": ms,
+            "roofline": {"bound": "tensor", "achieved": ach, "peak": tpeak, "unit": "TFLOP/s",
+                         "frac": ach / tpeak, "traffic": None,
+                         "kernel": "whole mmshift_coverage call (pack, softmax pass, merge, mass pass, "
+                                   "coverage)",
+                         "note": "algorithmic flops of the decode queries only; each query is its own "
+                                 "group, padded from r to 16 rows per KV head"}}
 
 
 class PreStep:
@@ -642,6 +718,11 @@ def run_gpu(args, wl):
                 "frac": achieved / peak, "traffic": None, "kernel": dom,
                 "peak_kind": f"fp32 FMA: {SM_COUNT} SMs x {FP32_LANES_PER_SM} lanes x 2 flop x {mhz:.0f} MHz"}
 
+    coverage = None
+    if args.coverage:
+        coverage = measure_coverage(args, wl, shape, K, Q, out_idx, stream, wl.seed + 104729 * (rank + 1), M,
+                                    float(peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])))
+
     cpu = None
     if rank == 0 and args.cpu_seconds > 0:
         rate, sample = oracle_sample_rate(wl, Kh, Vh, Qh, hyper, budget_s=args.cpu_seconds)
@@ -677,6 +758,7 @@ def run_gpu(args, wl):
         "clocks": clk,
         "gpu_launches": launches,
         "input_gen_s": gen_s,
+        **({"coverage": coverage} if coverage else {}),
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -700,6 +782,9 @@ def main(argv=None):
                          "(mmshift_prefill_stats + mmshift_select_with_stats); or over the prefill "
                          "hidden states with proxies projected by W_Q (mmshift_hidden_stats + "
                          "mmshift_build_hidden_proxies + mmshift_select)")
+    ap.add_argument("--coverage", type=int, default=32,
+                    help="decode queries per (layer, request) for the attention-mass coverage of "
+                         "the kept set (0 disables)")
     ap.add_argument("--d-model", type=int, default=0,
                     help="hidden size for --stats hidden (0: Hq * d, as in Qwen2.5-VL-7B)")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,

@@ -283,6 +283,24 @@ mmshift_status mmshift_select_with_stats(const mmshift_shape* s, const void* K, 
                                          void* out_V, const mmshift_debug* dbg, void* workspace,
                                          size_t workspace_bytes, mmshift_stream_t stream);
 
+/* Quality metric (Section 1, Fig. 1b): attention-mass coverage of a kept
+ * set. For decode query g of query head hq (dec_q [L, batch, Hq, n_dec, d]
+ * in the shape's dtype, the proxies_in layout), the softmax of
+ * scale * q.k_t over the T_b prompt keys of KV head h = hq / r, summed over
+ * the kept indices idx [L, R, Hkv] (e.g. mmshift_select's out_idx: indices
+ * in [0, T_b); others are skipped and reported by mmshift_poll_status) and
+ * averaged over the r query heads of h: cov [L][batch][Hkv][n_dec] float32.
+ * Steps 2-4 run with the decode queries as n_dec groups of one proxy (so the
+ * masses come from the same kernels as the selection's); Qwin supplies the
+ * anchor rows those kernels also compute. softmax_scale 0 = 1/sqrt(d);
+ * 1 <= n_dec <= 1024; workspace: mmshift_coverage_workspace_size() bytes. */
+mmshift_status mmshift_coverage_workspace_size(const mmshift_shape* s, int32_t n_dec,
+                                               size_t* bytes);
+mmshift_status mmshift_coverage(const mmshift_shape* s, const void* K, const void* Qwin,
+                                const void* dec_q, int32_t n_dec, float softmax_scale,
+                                const int32_t* idx, float* cov, void* workspace,
+                                size_t workspace_bytes, mmshift_stream_t stream);
+
 /* Allocation-free variant of mmshift_scores_topk.
  *
  * The paper has no counterpart: this entry point exists for callers that

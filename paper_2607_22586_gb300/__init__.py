@@ -14,4 +14,5 @@ from ._lib import (MMShiftError, Params, Shape, Debug, check, default_params,  #
                    mmshift_workspace_size, mmshift_prefill_stats, mmshift_prefill_stats_workspace_size,
                    mmshift_build_proxies_from_stats, mmshift_select_with_stats,
                    mmshift_hidden_stats_workspace_size, mmshift_hidden_stats,
-                   mmshift_hidden_proxies_workspace_size, mmshift_build_hidden_proxies)
+                   mmshift_hidden_proxies_workspace_size, mmshift_build_hidden_proxies,
+                   mmshift_coverage_workspace_size, mmshift_coverage)

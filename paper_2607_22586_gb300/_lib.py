@@ -36,6 +36,7 @@ EXPORTED = [
     "mmshift_build_proxies_from_stats", "mmshift_select_with_stats",
     "mmshift_hidden_stats_workspace_size", "mmshift_hidden_stats",
     "mmshift_hidden_proxies_workspace_size", "mmshift_build_hidden_proxies",
+    "mmshift_coverage_workspace_size", "mmshift_coverage",
 ]
 MMSHIFT_NOALLOC_SCRATCH_BYTES = 8 << 20
 
@@ -115,6 +116,11 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.mmshift_build_hidden_proxies.argtypes = [_SP, ctypes.c_int32, _VP, _VP, ctypes.c_int64, _VP,
                                                  _VP, _PP, _VP, _VP, ctypes.c_size_t, _VP]
     lib.mmshift_build_hidden_proxies.restype = st
+    lib.mmshift_coverage_workspace_size.argtypes = [_SP, ctypes.c_int32, ctypes.POINTER(ctypes.c_size_t)]
+    lib.mmshift_coverage_workspace_size.restype = st
+    lib.mmshift_coverage.argtypes = [_SP, _VP, _VP, _VP, ctypes.c_int32, ctypes.c_float, _VP, _VP, _VP,
+                                     ctypes.c_size_t, _VP]
+    lib.mmshift_coverage.restype = st
     lib.mmshift_proxy_mass.argtypes = [_SP, _VP, _VP, _VP, _PP, _VP, _VP, _VP, _VP, ctypes.c_size_t, _VP]
     lib.mmshift_proxy_mass.restype = st
     lib.mmshift_scores_topk.argtypes = [_SP, _PP, _VP, _VP, _VP, _VP, _VP, ctypes.c_size_t, _VP]
@@ -311,6 +317,22 @@ def mmshift_select_with_stats(shape, K, V, qwin, stats, params, out_idx, out_K, 
     return load_library().mmshift_select_with_stats(
         ctypes.byref(shape), _ptr(K), _ptr(V), _ptr(qwin), _ptr(stats), ctypes.byref(params),
         _ptr(out_idx), _ptr(out_K), _ptr(out_V), dbg, _ptr(workspace), workspace_bytes, _ptr(stream))
+
+
+
+def mmshift_coverage_workspace_size(shape: Shape, n_dec: int) -> int:
+    n = ctypes.c_size_t()
+    check(load_library().mmshift_coverage_workspace_size(ctypes.byref(shape), int(n_dec),
+                                                         ctypes.byref(n)),
+          "mmshift_coverage_workspace_size")
+    return n.value
+
+
+def mmshift_coverage(shape, K, qwin, dec_q, n_dec, softmax_scale, idx, cov, workspace,
+                     workspace_bytes, stream=None) -> int:
+    return load_library().mmshift_coverage(ctypes.byref(shape), _ptr(K), _ptr(qwin), _ptr(dec_q),
+                                           int(n_dec), float(softmax_scale), _ptr(idx), _ptr(cov),
+                                           _ptr(workspace), workspace_bytes, _ptr(stream))
 
 
 def mmshift_poll_status(workspace, stream=None) -> int:

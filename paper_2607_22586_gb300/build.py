@@ -20,7 +20,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libmmshift.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 SOURCES = ["api.cu", "proxy.cu", "score_simt.cu", "score_umma.cu", "select.cu", "stats.cu",
-           "hidden.cu", "noalloc.cu"]
+           "hidden.cu", "coverage.cu", "noalloc.cu"]
 
 
 def _nvcc() -> str:

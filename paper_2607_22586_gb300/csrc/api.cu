@@ -580,6 +580,49 @@ mmshift_status mmshift_select_with_stats(const mmshift_shape* s, const void* K, 
                      workspace_bytes, stream);
 }
 
+// Hyper-parameters under which steps 2-4 give the coverage masses: the
+// decode queries are the proxies, one per group.
+static mmshift_status coverage_params(int32_t n_dec, float softmax_scale, mmshift_params* p) {
+  if (n_dec < 1 || n_dec > 1024) return MMSHIFT_ERR_INVALID_ARG;
+  if (!(softmax_scale >= 0.f) || !std::isfinite(softmax_scale)) return MMSHIFT_ERR_INVALID_ARG;
+  mmshift_default_params(p);
+  p->n_proxies = n_dec;
+  p->n_groups = n_dec;
+  p->softmax_scale = softmax_scale;
+  p->score_mode = MMSHIFT_SCORE_MASS;
+  return MMSHIFT_OK;
+}
+
+mmshift_status mmshift_coverage_workspace_size(const mmshift_shape* s, int32_t n_dec,
+                                               size_t* bytes) {
+  mmshift_params p;
+  const mmshift_status st = coverage_params(n_dec, 0.f, &p);
+  if (st != MMSHIFT_OK) return st;
+  return mmshift_workspace_size(s, &p, bytes);
+}
+
+mmshift_status mmshift_coverage(const mmshift_shape* s, const void* K, const void* Qwin,
+                                const void* dec_q, int32_t n_dec, float softmax_scale,
+                                const int32_t* idx, float* cov, void* workspace,
+                                size_t workspace_bytes, mmshift_stream_t stream) {
+  mmshift_params p;
+  mmshift_status st = coverage_params(n_dec, softmax_scale, &p);
+  if (st != MMSHIFT_OK) return st;
+  Problem P;
+  if ((st = prepare(s, &p, &P)) != MMSHIFT_OK) return st;
+  if (!K || !Qwin || !dec_q || !idx || !cov) return MMSHIFT_ERR_INVALID_ARG;
+  P.use_umma = choose_umma(P, K);
+  P.part_slots = P.use_umma ? kUmmaPartSlots : 1;
+  Buffers bf;
+  if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
+  bf.proxies_in = dec_q;
+  bf.mass = nullptr;
+  const cudaStream_t cs = (cudaStream_t)stream;
+  if ((st = run_mass(P, bf, K, Qwin, cs)) != MMSHIFT_OK) return st;
+  const cudaError_t e = launch_coverage(P, bf, idx, cov, cs);
+  return e == cudaSuccess ? MMSHIFT_OK : cuda_fail(e);
+}
+
 mmshift_status mmshift_poll_status(void* workspace, mmshift_stream_t stream) {
   if (!workspace) return MMSHIFT_ERR_INVALID_ARG;
   cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);

@@ -177,6 +177,9 @@ bool make_tmap_bf16_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d
 bool tmap_encoder_available();
 int umma_launches(const Problem& P);
 cudaError_t launch_merge(const Problem& P, const Buffers& bf, cudaStream_t st);
+// Attention-mass coverage of the kept set idx from the group masses in bf.
+cudaError_t launch_coverage(const Problem& P, const Buffers& bf, const int32_t* idx, float* cov,
+                            cudaStream_t st);
 cudaError_t launch_cover(const Problem& P, const Buffers& bf, cudaStream_t st);
 cudaError_t launch_mass_sum(const Problem& P, const Buffers& bf, cudaStream_t st);
 cudaError_t launch_topk(const Problem& P, const Buffers& bf, cudaStream_t st,

@@ -295,6 +295,22 @@ def make_decode_queries(wl: Workload, layer: int, li: LayerInputs, n_dec: int,
     return out
 
 
+def make_kept_indices(wl: Workload, seed: int) -> np.ndarray:
+    """A seeded kept set in the output layout [R, Hkv] int32: per request
+    and KV head min(C_b, T_b) distinct ascending indices, always T_b - 1 (the
+    shape a selection produces, for tests that need one the oracle can take)."""
+    rng = np.random.Generator(np.random.Philox(key=[seed, 0x4B455054]))
+    rows = []
+    for t_len, c in zip(wl.seq_lens, wl.budgets):
+        keep = min(c, t_len)
+        blk = np.empty((keep, wl.n_kv_heads), dtype=np.int32)
+        for h in range(wl.n_kv_heads):
+            rest = rng.choice(t_len - 1, size=keep - 1, replace=False) if keep > 1 else np.zeros(0, int)
+            blk[:, h] = np.sort(np.concatenate([rest, [t_len - 1]]))
+        rows.append(blk)
+    return np.concatenate(rows)
+
+
 def make_proxies(wl: Workload, n_proxies: int, layer: int, scale: float = 8.0,
                  seed_tag: int = 0x50524F58) -> np.ndarray:
     """Seeded stand-alone proxy set [B, Hq, N_p, d] (dtype-exact float32).

@@ -149,3 +149,29 @@ def test_hidden_entries_validation_before_any_launch():
     w2 = M.mmshift_hidden_proxies_workspace_size(s2, dm, p)
     assert call(shape=s2, wq_layer_stride=8 * 128 * dm - 8, workspace_bytes=w2) == L.MMSHIFT_ERR_INVALID_ARG
     assert call(params=M.default_params(n_proxies=0, n_groups=0)) == L.MMSHIFT_OK   # nothing to do
+
+
+def test_coverage_validation_before_any_launch():
+    s = _shape()
+    n = M.mmshift_coverage_workspace_size(s, 16)
+    assert n > 0 and n % 256 == 0
+    fake = 1 << 40
+    args = [fake, fake, fake, 16, 0.0, fake, fake, fake, n]
+    bad = list(args)
+    bad[3] = 0
+    assert M.mmshift_coverage(s, *bad) == L.MMSHIFT_ERR_INVALID_ARG          # no decode queries
+    bad = list(args)
+    bad[3] = 1025
+    assert M.mmshift_coverage(s, *bad) == L.MMSHIFT_ERR_INVALID_ARG          # more than 1024
+    bad = list(args)
+    bad[4] = -1.0
+    assert M.mmshift_coverage(s, *bad) == L.MMSHIFT_ERR_INVALID_ARG          # negative scale
+    for i in (0, 1, 2, 5, 6):
+        bad = list(args)
+        bad[i] = None
+        assert M.mmshift_coverage(s, *bad) == L.MMSHIFT_ERR_INVALID_ARG, i
+    bad = list(args)
+    bad[8] = n - 256
+    assert M.mmshift_coverage(s, *bad) == L.MMSHIFT_ERR_WORKSPACE
+    with pytest.raises(L.MMShiftError):
+        M.mmshift_coverage_workspace_size(s, 0)
