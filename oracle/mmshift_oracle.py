@@ -34,7 +34,7 @@ __all__ = [
     "proxy_normals", "window_stats", "prefill_stats", "rope_rotate", "round_to",
     "build_proxies", "build_proxies_from_stats", "hidden_normals", "hidden_proxies",
     "softmax_rows", "group_masses", "anchor_attention", "cover_sets", "votes",
-    "scores", "select_topk", "gather", "attention_coverage", "select_request", "select",
+    "scores", "select_topk", "select_topk_heads", "gather", "attention_coverage", "select_request", "select",
 ]
 
 # ---------------------------------------------------------------------------
@@ -374,11 +374,35 @@ def select_topk(s: np.ndarray, budget: int) -> np.ndarray:
     return np.sort(kept).astype(np.int64)
 
 
+def select_topk_heads(s: np.ndarray, head_budgets: Sequence[int], capacity: int):
+    """Selection with a budget per KV head (§3.1: the budget C_{l,h} is set per
+    layer and KV head; §4.1 uses one value everywhere; §4.3 pairs the method
+    with allocators that spread budgets over layers and heads). Head h keeps
+    select_topk(s[h], C_h). Reading: every head's rows are padded to the
+    request's capacity min(C_max, T) with -1, C_max >= C_h >= 1 being the
+    request's largest budget. s: [Hkv, T] -> (idx [min(C_max, T), Hkv] int64,
+    counts [Hkv] = min(C_h, T))."""
+    hkv, t_len = s.shape
+    rows = min(capacity, t_len)
+    idx = np.full((rows, hkv), -1, dtype=np.int64)
+    counts = np.zeros(hkv, dtype=np.int64)
+    for h in range(hkv):
+        c = int(head_budgets[h])
+        assert 1 <= c <= capacity
+        kept = select_topk(s[h], c)
+        idx[:kept.shape[0], h] = kept
+        counts[h] = kept.shape[0]
+    return idx, counts
+
+
 def gather(keys: np.ndarray, values: np.ndarray, idx: np.ndarray):
-    """Compacted cache (Appendix B): row c of KV head h is token idx[c, h].
+    """Compacted cache (Appendix B): row c of KV head h is token idx[c, h];
+    padding rows (idx -1, per-head budgets) are zero.
     keys/values: [T, Hkv, d]; idx: [C', Hkv] -> two [C', Hkv, d] arrays."""
     h = np.arange(idx.shape[1])[None, :]
-    return keys[idx, h], values[idx, h]
+    pad = (idx < 0)[..., None]
+    safe = np.where(idx < 0, 0, idx)
+    return np.where(pad, 0.0, keys[safe, h]), np.where(pad, 0.0, values[safe, h])
 
 
 # ---------------------------------------------------------------------------
@@ -415,15 +439,18 @@ def select_request(keys, values, qwin, budget: int, *, n_proxies=512, n_groups=3
                    gamma=10.0, tau=0.95, lam=1.0, seed=0, layer_id=0, b=0,
                    score_mode=SCORE_VOTE, softmax_scale=0.0, rope_theta=0.0,
                    rope_pos_offset=0, dtype=BF16, proxies=None,
-                   qfull=None) -> Dict[str, np.ndarray]:
+                   qfull=None, head_budgets=None) -> Dict[str, np.ndarray]:
     """Algorithm 1 for one request of one layer.
 
     keys/values: [T, Hkv, d]; qwin: [W, Hq, d] (its last row is the last real
     prefill query). ``proxies`` ([Hq, N_p, d]) replaces the sampled proxies
     when given. ``qfull`` ([T, Hq, d], all prompt queries), when given, is the
     source of the proxies' statistics (prefill_stats) instead of the window.
+    ``head_budgets`` ([Hkv], each in [1, budget]) gives every KV head its own
+    budget (select_topk_heads); ``budget`` is then the request's largest.
     Returns proxies, group masses, anchor, mass, scores, indices ([C', Hkv],
-    ascending per head) and the gathered cache.
+    ascending per head, -1 padded with head budgets), the kept count per head
+    and the gathered cache.
     """
     keys = np.asarray(keys, dtype=np.float64)
     values = np.asarray(values, dtype=np.float64)
@@ -445,10 +472,14 @@ def select_request(keys, values, qwin, budget: int, *, n_proxies=512, n_groups=3
     alpha = anchor_attention(qwin[-1], keys, scale)                # [Hkv, T]
     mass = abar.sum(axis=1)                                         # [Hkv, T]
     s = np.stack([scores(score_mode, abar[h], alpha[h], tau, lam) for h in range(hkv)])
-    idx = np.stack([select_topk(s[h], budget) for h in range(hkv)], axis=1)
+    if head_budgets is None:
+        idx = np.stack([select_topk(s[h], budget) for h in range(hkv)], axis=1)
+        count = np.full(hkv, idx.shape[0], dtype=np.int64)
+    else:
+        idx, count = select_topk_heads(s, head_budgets, budget)
     out_k, out_v = gather(keys, values, idx)
     return dict(proxies=proxies, group_mass=abar, anchor=alpha, mass=mass,
-                scores=s, idx=idx, out_k=out_k, out_v=out_v)
+                scores=s, idx=idx, count=count, out_k=out_k, out_v=out_v)
 
 
 def select(keys, values, qwin, cu_seqlens: Sequence[int], budgets: Sequence[int],

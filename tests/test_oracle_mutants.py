@@ -194,6 +194,26 @@ def _coverage_renormalised_on_kept(keys, dec_queries, idx, scale):
     return out
 
 
+def _topk_heads_capacity_everywhere(s, head_budgets, capacity):
+    hkv, t_len = s.shape
+    idx = np.stack([O.select_topk(s[h], capacity) for h in range(hkv)], axis=1)
+    return idx, np.full(hkv, idx.shape[0], dtype=np.int64)
+
+
+def _topk_heads_drops_last_token(s, head_budgets, capacity):
+    hkv, t_len = s.shape
+    rows = min(capacity, t_len)
+    idx = np.full((rows, hkv), -1, dtype=np.int64)
+    counts = np.zeros(hkv, dtype=np.int64)
+    for h in range(hkv):
+        c = min(int(head_budgets[h]), t_len)
+        order = np.lexsort((np.arange(t_len), -s[h]))
+        kept = np.sort(order[:c])
+        idx[:c, h] = kept
+        counts[h] = c
+    return idx, counts
+
+
 MUTANTS = {
     "std_ddof0": ("window_stats", _window_stats_ddof0),
     "prefill_std_ddof0": ("prefill_stats", _prefill_stats_ddof0),
@@ -217,6 +237,8 @@ MUTANTS = {
     "coverage_modulo_heads": ("attention_coverage", _coverage_modulo_heads),
     "coverage_no_scale": ("attention_coverage", _coverage_no_scale),
     "coverage_renormalised_on_kept": ("attention_coverage", _coverage_renormalised_on_kept),
+    "head_budgets_ignored": ("select_topk_heads", _topk_heads_capacity_everywhere),
+    "head_budgets_drop_last_token": ("select_topk_heads", _topk_heads_drops_last_token),
 }
 
 

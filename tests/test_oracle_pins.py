@@ -188,6 +188,34 @@ def pin_attention_coverage(orc=O):
     assert np.all(cov[2:] > 1.0 - 1e-12)
 
 
+def pin_head_budgets(orc=O):
+    """Per-head budgets (§3.1's C_{l,h}): equal budgets reproduce the uniform
+    selection; each head keeps exactly min(C_h, T) tokens, its own top ones
+    (brute force over subsets: no other set of that size containing T-1 has
+    a larger score sum), the rest of its rows -1; a smaller budget keeps a
+    subset of a larger one's tokens; padded rows gather zeros."""
+    rng = np.random.default_rng(53)
+    hkv, t_len = 3, 10
+    s = rng.integers(0, 4, size=(hkv, t_len)).astype(np.float64) + rng.random((hkv, t_len)) * 0.5
+    idx_u = np.stack([orc.select_topk(s[h], 4) for h in range(hkv)], axis=1)
+    idx_e, cnt_e = orc.select_topk_heads(s, [4, 4, 4], 4)
+    assert np.array_equal(idx_u, idx_e) and np.array_equal(cnt_e, [4, 4, 4])
+    idx, cnt = orc.select_topk_heads(s, [1, 3, 6], 6)
+    assert idx.shape == (6, hkv) and np.array_equal(cnt, [1, 3, 6])
+    for h, c in enumerate([1, 3, 6]):
+        kept = idx[:c, h]
+        assert np.all(idx[c:, h] == -1) and kept[-1] == t_len - 1 and np.all(np.diff(kept) > 0)
+        best = max(sum(s[h][list(sub)]) for sub in itertools.combinations(range(t_len - 1), c - 1))
+        assert math.isclose(s[h][kept[:-1]].sum(), best, rel_tol=0, abs_tol=1e-12)
+    small, _ = orc.select_topk_heads(s, [2, 2, 2], 6)
+    assert set(idx[:1, 0]) <= set(small[:2, 0])
+    for h in (1, 2):
+        assert set(small[:2, h]) <= set(idx[:cnt[h], h])
+    keys = rng.normal(size=(t_len, hkv, 4))
+    ok, ov = orc.gather(keys, keys, idx)
+    assert np.all(ok[1:, 0] == 0.0) and np.array_equal(ok[:3, 1], keys[idx[:3, 1], 1])
+
+
 def pin_sampler_closed_form(orc=O):
     """Appendix A.2: for q ~ N(mu, Sigma), E[exp(q.k/sqrt d)] =
     exp(mu.k/sqrt d + k^T Sigma k / (2d)). With Sigma = diag((gamma*sigma)^2)
@@ -409,7 +437,7 @@ def pin_topk_bruteforce(orc=O):
 
 
 ALL_PINS = [pin_philox_vs_numpy, pin_normals_distribution, pin_window_stats, pin_prefill_stats,
-            pin_hidden_proxies, pin_attention_coverage,
+            pin_hidden_proxies, pin_attention_coverage, pin_head_budgets,
             pin_sampler_closed_form, pin_rope, pin_round_bf16, pin_mass_totals,
             pin_sigma_zero_single_query, pin_shift_and_permutation, pin_budget_ge_t,
             pin_lastattn, pin_uniform_keys, pin_cover_bruteforce, pin_topk_bruteforce]
