@@ -283,6 +283,27 @@ mmshift_status mmshift_select_with_stats(const mmshift_shape* s, const void* K, 
                                          void* out_V, const mmshift_debug* dbg, void* workspace,
                                          size_t workspace_bytes, mmshift_stream_t stream);
 
+/* Budgets per layer and KV head (Section 3.1 defines the budget C_{l,h} per
+ * layer and KV head; Section 4.3 pairs the selection with allocators that
+ * spread budgets over layers and heads). head_budgets: device
+ * [L][batch][Hkv] int32, C_{l,b,h} in [1, budgets[b]] (the shape's budgets
+ * are each request's capacity: they size the output rows; values outside are
+ * clamped and reported by mmshift_poll_status). Head h of request b keeps
+ * min(C_{l,b,h}, T_b) rows of out_idx (T_b - 1 and the top others, in
+ * ascending order); its remaining rows up to min(C_b, T_b) hold -1 and
+ * gather zero K/V rows. out_count (nullable): device [L][batch][Hkv] int32,
+ * the kept rows per head. Otherwise as mmshift_select / mmshift_topk. */
+mmshift_status mmshift_select_head_budgets(const mmshift_shape* s, const void* K, const void* V,
+                                           const void* Qwin, const void* proxies_in,
+                                           const int32_t* head_budgets, const mmshift_params* p,
+                                           int32_t* out_idx, int32_t* out_count, void* out_K,
+                                           void* out_V, const mmshift_debug* dbg, void* workspace,
+                                           size_t workspace_bytes, mmshift_stream_t stream);
+mmshift_status mmshift_topk_head_budgets(const mmshift_shape* s, const float* scores,
+                                         const int32_t* head_budgets, int32_t* out_idx,
+                                         int32_t* out_count, void* workspace,
+                                         size_t workspace_bytes, mmshift_stream_t stream);
+
 /* Quality metric (Section 1, Fig. 1b): attention-mass coverage of a kept
  * set. For decode query g of query head hq (dec_q [L, batch, Hq, n_dec, d]
  * in the shape's dtype, the proxies_in layout), the softmax of

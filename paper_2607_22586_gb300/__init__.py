@@ -15,4 +15,5 @@ from ._lib import (MMShiftError, Params, Shape, Debug, check, default_params,  #
                    mmshift_build_proxies_from_stats, mmshift_select_with_stats,
                    mmshift_hidden_stats_workspace_size, mmshift_hidden_stats,
                    mmshift_hidden_proxies_workspace_size, mmshift_build_hidden_proxies,
-                   mmshift_coverage_workspace_size, mmshift_coverage)
+                   mmshift_coverage_workspace_size, mmshift_coverage,
+                   mmshift_select_head_budgets, mmshift_topk_head_budgets)

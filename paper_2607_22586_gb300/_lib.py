@@ -37,6 +37,7 @@ EXPORTED = [
     "mmshift_hidden_stats_workspace_size", "mmshift_hidden_stats",
     "mmshift_hidden_proxies_workspace_size", "mmshift_build_hidden_proxies",
     "mmshift_coverage_workspace_size", "mmshift_coverage",
+    "mmshift_select_head_budgets", "mmshift_topk_head_budgets",
 ]
 MMSHIFT_NOALLOC_SCRATCH_BYTES = 8 << 20
 
@@ -121,6 +122,11 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.mmshift_coverage.argtypes = [_SP, _VP, _VP, _VP, ctypes.c_int32, ctypes.c_float, _VP, _VP, _VP,
                                      ctypes.c_size_t, _VP]
     lib.mmshift_coverage.restype = st
+    lib.mmshift_select_head_budgets.argtypes = [_SP, _VP, _VP, _VP, _VP, _VP, _PP, _VP, _VP, _VP, _VP,
+                                                ctypes.POINTER(Debug), _VP, ctypes.c_size_t, _VP]
+    lib.mmshift_select_head_budgets.restype = st
+    lib.mmshift_topk_head_budgets.argtypes = [_SP, _VP, _VP, _VP, _VP, _VP, ctypes.c_size_t, _VP]
+    lib.mmshift_topk_head_budgets.restype = st
     lib.mmshift_proxy_mass.argtypes = [_SP, _VP, _VP, _VP, _PP, _VP, _VP, _VP, _VP, ctypes.c_size_t, _VP]
     lib.mmshift_proxy_mass.restype = st
     lib.mmshift_scores_topk.argtypes = [_SP, _PP, _VP, _VP, _VP, _VP, _VP, ctypes.c_size_t, _VP]
@@ -333,6 +339,24 @@ def mmshift_coverage(shape, K, qwin, dec_q, n_dec, softmax_scale, idx, cov, work
     return load_library().mmshift_coverage(ctypes.byref(shape), _ptr(K), _ptr(qwin), _ptr(dec_q),
                                            int(n_dec), float(softmax_scale), _ptr(idx), _ptr(cov),
                                            _ptr(workspace), workspace_bytes, _ptr(stream))
+
+
+
+def mmshift_select_head_budgets(shape, K, V, qwin, proxies_in, head_budgets, params, out_idx,
+                                out_count, out_K, out_V, debug, workspace, workspace_bytes,
+                                stream=None) -> int:
+    dbg = ctypes.byref(debug) if debug is not None else None
+    return load_library().mmshift_select_head_budgets(
+        ctypes.byref(shape), _ptr(K), _ptr(V), _ptr(qwin), _ptr(proxies_in), _ptr(head_budgets),
+        ctypes.byref(params), _ptr(out_idx), _ptr(out_count), _ptr(out_K), _ptr(out_V), dbg,
+        _ptr(workspace), workspace_bytes, _ptr(stream))
+
+
+def mmshift_topk_head_budgets(shape, scores, head_budgets, out_idx, out_count, workspace,
+                              workspace_bytes, stream=None) -> int:
+    return load_library().mmshift_topk_head_budgets(
+        ctypes.byref(shape), _ptr(scores), _ptr(head_budgets), _ptr(out_idx), _ptr(out_count),
+        _ptr(workspace), workspace_bytes, _ptr(stream))
 
 
 def mmshift_poll_status(workspace, stream=None) -> int:

@@ -296,7 +296,9 @@ static mmshift_status select_impl(const mmshift_shape* s, const void* K, const v
                                   const void* Qwin, const void* proxies_in, const float* stats_in,
                                   const mmshift_params* p, int32_t* out_idx, void* out_K,
                                   void* out_V, const mmshift_debug* dbg, void* workspace,
-                                  size_t workspace_bytes, mmshift_stream_t stream) {
+                                  size_t workspace_bytes, mmshift_stream_t stream,
+                                  const int32_t* head_budgets = nullptr,
+                                  int32_t* out_count = nullptr) {
   Problem P;
   mmshift_status st = prepare(s, p, &P);
   if (st != MMSHIFT_OK) return st;
@@ -307,6 +309,8 @@ static mmshift_status select_impl(const mmshift_shape* s, const void* K, const v
   if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
   bf.proxies_in = proxies_in;
   bf.stats_in = stats_in;
+  bf.head_budget = head_budgets;
+  bf.out_count = out_count;
   if (dbg) {
     bf.proxies_out = dbg->proxies;
     if (dbg->group_mass && P.G) bf.gmass = dbg->group_mass;
@@ -547,6 +551,23 @@ mmshift_status mmshift_topk(const mmshift_shape* s, const float* scores, int32_t
   return e == cudaSuccess ? MMSHIFT_OK : cuda_fail(e);
 }
 
+mmshift_status mmshift_topk_head_budgets(const mmshift_shape* s, const float* scores,
+                                         const int32_t* head_budgets, int32_t* out_idx,
+                                         int32_t* out_count, void* workspace,
+                                         size_t workspace_bytes, mmshift_stream_t stream) {
+  Problem P;
+  mmshift_status st = prepare(s, nullptr, &P);
+  if (st != MMSHIFT_OK) return st;
+  if (!scores || !head_budgets || !out_idx) return MMSHIFT_ERR_INVALID_ARG;
+  Buffers bf;
+  if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
+  bf.scores = const_cast<float*>(scores);
+  bf.head_budget = head_budgets;
+  bf.out_count = out_count;
+  const cudaError_t e = launch_topk(P, bf, (cudaStream_t)stream, out_idx, true);
+  return e == cudaSuccess ? MMSHIFT_OK : cuda_fail(e);
+}
+
 mmshift_status mmshift_gather(const mmshift_shape* s, const void* K, const void* V,
                               const int32_t* idx, void* out_K, void* out_V,
                               void* workspace, size_t workspace_bytes,
@@ -568,6 +589,17 @@ mmshift_status mmshift_select(const mmshift_shape* s, const void* K, const void*
                               size_t workspace_bytes, mmshift_stream_t stream) {
   return select_impl(s, K, V, Qwin, proxies_in, nullptr, p, out_idx, out_K, out_V, dbg,
                      workspace, workspace_bytes, stream);
+}
+
+mmshift_status mmshift_select_head_budgets(const mmshift_shape* s, const void* K, const void* V,
+                                           const void* Qwin, const void* proxies_in,
+                                           const int32_t* head_budgets, const mmshift_params* p,
+                                           int32_t* out_idx, int32_t* out_count, void* out_K,
+                                           void* out_V, const mmshift_debug* dbg, void* workspace,
+                                           size_t workspace_bytes, mmshift_stream_t stream) {
+  if (!head_budgets) return MMSHIFT_ERR_INVALID_ARG;
+  return select_impl(s, K, V, Qwin, proxies_in, nullptr, p, out_idx, out_K, out_V, dbg, workspace,
+                     workspace_bytes, stream, head_budgets, out_count);
 }
 
 mmshift_status mmshift_select_with_stats(const mmshift_shape* s, const void* K, const void* V,

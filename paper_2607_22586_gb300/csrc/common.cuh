@@ -19,6 +19,7 @@ constexpr int kUmmaPartSlots = 4; // softmax partials per (row, split) of the te
 enum : int {
   kStatusTimeout = 1,   // a bounded wait gave up
   kStatusBadIndex = 2,  // gather saw an index outside [0, T_b)
+  kStatusBadBudget = 4, // a per-head budget outside [1, C_b] (clamped)
 };
 
 struct ReqInfo {
@@ -69,6 +70,8 @@ struct Buffers {
   void* proxies_out;  // [L][B][Hq][Np][d] or null
   const void* proxies_in; // [L][B][Hq][Np][d] or null
   const float* stats_in;  // [L][B][2][Hq][d] mean / std of the proxies, or null (window's)
+  const int32_t* head_budget; // [L][B][Hkv] budgets C_{l,b,h} in [1, C_b], or null (C_b for all)
+  int32_t* out_count;         // [L][B][Hkv] kept rows per head, or null
 };
 
 // Whole-prefill statistics job (stats.cu).

@@ -430,7 +430,18 @@ __global__ void __launch_bounds__(NT, 1) topk_kernel(Problem P, Buffers bf, int3
   }
   __syncthreads();
   int32_t* out = out_idx + ((size_t)l * P.R + R.out_off) * P.Hkv + h;
-  const int keep = R.keep;
+  int keep = R.keep;
+  if (bf.head_budget) {
+    // this head's own budget; its rows past the kept ones are padding (-1)
+    int c = bf.head_budget[((size_t)l * P.B + b) * P.Hkv + h];
+    if (c < 1 || c > R.budget) {
+      if (tid == 0) set_status(bf.status, kStatusBadBudget);
+      c = min(max(c, 1), R.budget);
+    }
+    keep = min(c, n);
+    for (int i = keep + tid; i < R.keep; i += NT) out[(size_t)i * P.Hkv] = -1;
+  }
+  if (bf.out_count && tid == 0) bf.out_count[((size_t)l * P.B + b) * P.Hkv + h] = keep;
   if (keep >= n) {
     for (int i = tid; i < n; i += NT) out[(size_t)i * P.Hkv] = i;
     return;
@@ -502,9 +513,10 @@ __global__ void __launch_bounds__(256) gather_kernel(Problem P, Buffers bf, cons
   uint4* dk = (uint4*)(oK + (((size_t)l * P.R * P.Hkv + q) * ROWB)) + part;
   uint4* dv = (uint4*)(oV + (((size_t)l * P.R * P.Hkv + q) * ROWB)) + part;
   if (t < 0 || t >= R.t_len) {
+    // zero rows: padding of a head with its own smaller budget (-1), or a bad index
     *dk = make_uint4(0, 0, 0, 0);
     *dv = make_uint4(0, 0, 0, 0);
-    if (part == 0) set_status(bf.status, kStatusBadIndex);
+    if (part == 0 && !(bf.head_budget && t == -1)) set_status(bf.status, kStatusBadIndex);
     return;
   }
   const size_t src = (size_t)l * P.ls_kv * esz + (((size_t)R.tok_off + t) * P.Hkv + h) * ROWB;
