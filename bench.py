@@ -390,15 +390,33 @@ def hyper_for(args, wl):
     return dict(n_proxies=512, n_groups=32, gamma=10.0, tau=float(np.float32(0.95)), lam=1.0, seed=0)
 
 
-def algorithmic(wl, hyper):
+def pyramid_budgets(wl):
+    """Per-(layer, KV head) budgets [L, B, Hkv] shaped like a pyramid
+    allocation: layer l of L gets C * (1.5 - l / (L - 1)) (1.5 C at the
+    bottom, C / 2 at the top, C on average), equal across heads."""
+    L = wl.n_layers
+    hb = np.empty((L, wl.batch, wl.n_kv_heads), dtype=np.int32)
+    for l in range(L):
+        f = 1.5 - (l / (L - 1) if L > 1 else 0.5)
+        for b, c in enumerate(wl.budgets):
+            hb[l, b, :] = max(1, int(round(c * f)))
+    return hb
+
+
+def algorithmic(wl, hyper, head_budgets=None):
     """Per step: HBM bytes (K read once + K/V gathered read+write) and the
     logits of one softmax pass (2 d flops per (proxy row, key))."""
     esz = 2 if wl.dtype == S.BF16 else 4
     L, hkv, d = wl.n_layers, wl.n_kv_heads, wl.head_dim
     T = wl.total_tokens
-    keep = sum(min(c, t) for c, t in zip(wl.budgets, wl.seq_lens))
     k_read = L * T * hkv * d * esz
-    gather = 4 * L * keep * hkv * d * esz
+    if head_budgets is None:
+        keep = sum(min(c, t) for c, t in zip(wl.budgets, wl.seq_lens))
+        gather = 4 * L * keep * hkv * d * esz
+    else:
+        kept = sum(int(min(head_budgets[l, b, h], t)) for l in range(L)
+                   for b, t in enumerate(wl.seq_lens) for h in range(hkv))
+        gather = 4 * kept * d * esz
     r = wl.n_q_heads // hkv
     rows = hyper["n_proxies"] * r + r       # proxies of the r query heads + anchor rows
     pass_flops = 2.0 * d * rows * T * hkv * L
@@ -533,8 +551,11 @@ def run_gpu(args, wl):
 
     L = wl.n_layers
     T = wl.total_tokens
+    hb_host = pyramid_budgets(wl) if args.head_budgets == "pyramid" else None
+    capacity = wl.budgets if hb_host is None else tuple(int(hb_host[:, b].max())
+                                                        for b in range(wl.batch))
     shape = M.make_shape(wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.window,
-                         0 if wl.dtype == S.BF16 else 1, wl.cu_seqlens(), wl.budgets, n_layers=L,
+                         0 if wl.dtype == S.BF16 else 1, wl.cu_seqlens(), capacity, n_layers=L,
                          layer_stride_kv=T * wl.n_kv_heads * wl.head_dim,
                          layer_stride_q=wl.batch * wl.window * wl.n_q_heads * wl.head_dim)
     params = M.default_params(n_proxies=hyper["n_proxies"], n_groups=hyper["n_groups"],
@@ -552,8 +573,14 @@ def run_gpu(args, wl):
     if args.stats != "window":
         pre = PreStep(args.stats, wl, shape, params, K, Q, wl.seed + 7919 * (rank + 1), d_model, M)
 
+    hb_dev = torch.from_numpy(hb_host).to(dev) if hb_host is not None else None
+
     def select(Kx, Vx, Qx, Xx, dbg=None, sev=None):
-        if pre is None:
+        if hb_dev is not None:
+            M.check(M.mmshift_select_head_budgets(shape, Kx, Vx, Qx, None, hb_dev, params, out_idx,
+                                                  None, out_k, out_v, dbg, ws, ws_bytes, stream),
+                    "mmshift_select_head_budgets")
+        elif pre is None:
             M.check(M.mmshift_select(shape, Kx, Vx, Qx, None, params, out_idx, out_k, out_v, dbg,
                                      ws, ws_bytes, stream), "mmshift_select")
         elif pre.kind == "prefill":
@@ -662,7 +689,7 @@ def run_gpu(args, wl):
         h2d += X_pin.numel() * X_pin.element_size()
     d2h = sum(t.numel() * t.element_size() for t in (idx_h, ok_h, ov_h))
 
-    bytes_step, k_read, pass_flops = algorithmic(wl, hyper)
+    bytes_step, k_read, pass_flops = algorithmic(wl, hyper, hb_host)
     extra_roofs = {}
     if pre:
         # algorithmic bytes of the statistics pass: every prompt query (or
@@ -741,7 +768,7 @@ def run_gpu(args, wl):
                    "window": wl.window, "budgets": list(wl.budgets), "proxies": args.proxies,
                    "n_proxies": hyper["n_proxies"], "n_groups": hyper["n_groups"],
                    "gamma": hyper["gamma"], "tau": hyper["tau"], "lambda": hyper["lam"],
-                   "stats": args.stats,
+                   "stats": args.stats, "head_budgets": args.head_budgets,
                    **({"d_model": d_model} if args.stats == "hidden" else {}),
                    "l2": "inputs (K+V %.2f GB) larger than L2; no flush" % (2 * k_read / 1e9),
                    "parallelism": f"replicas x{world}"},
@@ -782,6 +809,10 @@ def main(argv=None):
                          "(mmshift_prefill_stats + mmshift_select_with_stats); or over the prefill "
                          "hidden states with proxies projected by W_Q (mmshift_hidden_stats + "
                          "mmshift_build_hidden_proxies + mmshift_select)")
+    ap.add_argument("--head-budgets", choices=["uniform", "pyramid"], default="uniform",
+                    help="budget per (layer, KV head): uniform C, or pyramid-shaped (1.5 C at the "
+                         "first layer to C/2 at the last, C on average) through "
+                         "mmshift_select_head_budgets")
     ap.add_argument("--coverage", type=int, default=32,
                     help="decode queries per (layer, request) for the attention-mass coverage of "
                          "the kept set (0 disables)")

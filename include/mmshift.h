@@ -309,7 +309,8 @@ mmshift_status mmshift_topk_head_budgets(const mmshift_shape* s, const float* sc
  * in the shape's dtype, the proxies_in layout), the softmax of
  * scale * q.k_t over the T_b prompt keys of KV head h = hq / r, summed over
  * the kept indices idx [L, R, Hkv] (e.g. mmshift_select's out_idx: indices
- * in [0, T_b); others are skipped and reported by mmshift_poll_status) and
+ * in [0, T_b); -1 marks padding rows and is skipped; other values are
+ * skipped and reported by mmshift_poll_status) and
  * averaged over the r query heads of h: cov [L][batch][Hkv][n_dec] float32.
  * Steps 2-4 run with the decode queries as n_dec groups of one proxy (so the
  * masses come from the same kernels as the selection's); Qwin supplies the

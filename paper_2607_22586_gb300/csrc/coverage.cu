@@ -43,7 +43,7 @@ __global__ void __launch_bounds__(kCovThreads) coverage_kernel(Problem P, const 
   for (int c = threadIdx.x; c < R.keep; c += kCovThreads) {
     const int t = id[(size_t)c * P.Hkv];
     if ((unsigned)t < (unsigned)R.t_len) kept += row[t];
-    else bad = true;
+    else if (t != -1) bad = true;   // -1: padding row of a head with a smaller budget
   }
   for (int t = threadIdx.x; t < R.t_len; t += kCovThreads) tot += row[t];
   if (bad) set_status(status, kStatusBadIndex);
