@@ -139,8 +139,45 @@ __device__ __forceinline__ void digit_histogram(const KeySrc& get, int n, uint32
   unsigned long long tot = 0;
   uint32_t kmax = 0;
   const float scale = pow2f(shift);
+  auto count = [&](uint32_t k, bool valid) {
+    const bool take = valid && (k >> hs) == (prefix >> hs);
+    if (!first && !__any_sync(0xffffffffu, take)) return;
+    if (take) {
+      const uint32_t d = (k >> sh) & dmask;
+      atomicAdd(&hn[d], 1u);
+      if (WEIGHTED) {
+        const unsigned long long wt = fx_weight(k, scale);
+        if (first) { tot += wt; kmax = max(kmax, k); }
+        add_weight(&hlo[d], &hhi[d], wt);
+      }
+    }
+  };
+  int done = 0;
+  if (!get.smem && (reinterpret_cast<uintptr_t>(get.gmem) & 15) == 0) {
+    // 16-byte loads of four keys, four loads in flight per thread
+    constexpr int U4 = 4;
+    const float4* g4 = reinterpret_cast<const float4*>(get.gmem);
+    const int n4 = n >> 2;
+    for (int base = 0; base < n4; base += U4 * NTH) {
+      float4 f[U4];
+#pragma unroll
+      for (int j = 0; j < U4; ++j) {
+        const int i4 = base + j * NTH + tid;
+        f[j] = i4 < n4 ? __ldg(g4 + i4) : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int j = 0; j < U4; ++j) {
+        const bool valid = base + j * NTH + tid < n4;
+        count(nonneg_key(f[j].x), valid);
+        count(nonneg_key(f[j].y), valid);
+        count(nonneg_key(f[j].z), valid);
+        count(nonneg_key(f[j].w), valid);
+      }
+    }
+    done = n4 << 2;
+  }
   constexpr int U = 8;  // independent loads in flight per thread
-  for (int base = 0; base < n; base += U * NTH) {
+  for (int base = done; base < n; base += U * NTH) {
     uint32_t kk[U];
 #pragma unroll
     for (int j = 0; j < U; ++j) {
@@ -148,21 +185,7 @@ __device__ __forceinline__ void digit_histogram(const KeySrc& get, int n, uint32
       kk[j] = i < n ? get(i) : 0u;
     }
 #pragma unroll
-    for (int j = 0; j < U; ++j) {
-      const int i = base + j * NTH + tid;
-      const uint32_t k = kk[j];
-      const bool take = i < n && (k >> hs) == (prefix >> hs);
-      if (!first && !__any_sync(0xffffffffu, take)) continue;
-      if (take) {
-        const uint32_t d = (k >> sh) & dmask;
-        atomicAdd(&hn[d], 1u);
-        if (WEIGHTED) {
-          const unsigned long long wt = fx_weight(k, scale);
-          if (first) { tot += wt; kmax = max(kmax, k); }
-          add_weight(&hlo[d], &hhi[d], wt);
-        }
-      }
-    }
+    for (int j = 0; j < U; ++j) count(kk[j], base + j * NTH + tid < n);
   }
   if (WEIGHTED && first) {
     for (int off = 16; off; off >>= 1) {
