@@ -11,6 +11,8 @@
 //     (group g holds the g-th slice of every query head of the KV head), the
 //     last window query of each query head as anchor rows, zero padding;
 //   - optionally the caller-layout copy [Hq][N][d].
+#include <algorithm>
+
 #include "common.cuh"
 #include "rng.cuh"
 
@@ -38,12 +40,14 @@ __device__ __forceinline__ void store4(float* dst, float a, float b, float c, fl
   *reinterpret_cast<float4*>(dst) = make_float4(a, b, c, d);
 }
 
-// Proxies of one query head are spread over kProxyChunks CTAs.
+// Proxies of one query head are spread over up to kProxyChunks CTAs, about
+// 1024 Philox draws each (few proxies: one CTA per query head).
 constexpr int kProxyChunks = 8;
 
 template <typename T, int D>
-__global__ void __launch_bounds__(256) proxy_pack_kernel(Problem P, Buffers bf, const T* qwin) {
-  const int hq = blockIdx.x / kProxyChunks, chunk = blockIdx.x % kProxyChunks;
+__global__ void __launch_bounds__(256) proxy_pack_kernel(Problem P, Buffers bf, const T* qwin,
+                                                         int nch) {
+  const int hq = blockIdx.x / nch, chunk = blockIdx.x % nch;
   const int b = blockIdx.y, l = blockIdx.z;
   const int h = hq / P.r, j = hq - h * P.r;
   __shared__ float mu[D], sg[D], rc[D / 2], rs[D / 2];
@@ -109,7 +113,7 @@ __global__ void __launch_bounds__(256) proxy_pack_kernel(Problem P, Buffers bf, 
   const T* pin = bf.proxies_in ? (const T*)bf.proxies_in + user_off : nullptr;
   T* pout = bf.proxies_out ? (T*)bf.proxies_out + user_off : nullptr;
   constexpr int NQ8 = D / 8;  // threads per proxy: dims [4qq, 4qq+4) and [D/2+4qq, +4)
-  const int per = (P.Np + kProxyChunks - 1) / kProxyChunks;
+  const int per = (P.Np + nch - 1) / nch;
   const int i0 = chunk * per, i1 = min(P.Np, i0 + per);
   // independent iterations unrolled so several Philox chains are in flight
 #pragma unroll 4
@@ -180,8 +184,10 @@ __global__ void __launch_bounds__(256) proxy_pack_kernel(Problem P, Buffers bf, 
 
 template <typename T, int D>
 cudaError_t launch_t(const Problem& P, const Buffers& bf, cudaStream_t st, const void* qwin) {
-  dim3 grid(P.Hq * kProxyChunks, P.B, P.L);
-  proxy_pack_kernel<T, D><<<grid, 256, 0, st>>>(P, bf, (const T*)qwin);
+  const int draws = P.Np * (D / 8);
+  const int nch = draws <= 0 ? 1 : std::min(kProxyChunks, (draws + 1023) / 1024);
+  dim3 grid(P.Hq * nch, P.B, P.L);
+  proxy_pack_kernel<T, D><<<grid, 256, 0, st>>>(P, bf, (const T*)qwin, nch);
   return cudaGetLastError();
 }
 

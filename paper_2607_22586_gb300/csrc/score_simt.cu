@@ -121,9 +121,17 @@ __global__ void merge_kernel(Problem P, Buffers bf) {
   float m = -INFINITY, z = 0.f;
   const float2* src =
       bf.part + (((size_t)l * P.Hkv + h) * P.total_splits + R.split_off) * P.part_slots * P.Prows_pad + p;
-  for (int s = 0; s < R.nsplit * P.part_slots; ++s) {
-    const float2 v = src[(size_t)s * P.Prows_pad];
-    merge_ms(m, z, v.x, v.y);
+  // partials merged in split order; eight loads issued ahead of the merges
+  const int ns = R.nsplit * P.part_slots;
+  constexpr int A = 8;
+  for (int s0 = 0; s0 < ns; s0 += A) {
+    float2 v[A];
+#pragma unroll
+    for (int u = 0; u < A; ++u)
+      v[u] = s0 + u < ns ? src[(size_t)(s0 + u) * P.Prows_pad] : make_float2(-INFINITY, 0.f);
+#pragma unroll
+    for (int u = 0; u < A; ++u)
+      if (s0 + u < ns) merge_ms(m, z, v[u].x, v[u].y);
   }
   const bool valid = row_kind(P, p).group >= 0;
   bf.cvals[(((size_t)l * P.B + b) * P.Hkv + h) * P.Prows_pad + p] =
