@@ -20,6 +20,8 @@ class KVSelector:
             raise ValueError(f"unsupported dtype {dtype}")
         self.dtype = dtype
         self.device = torch.device(device)
+        if self.device.type == "cuda" and self.device.index is None:
+            self.device = torch.device("cuda", torch.cuda.current_device())
         total = int(cu_seqlens[-1])
         self.total_tokens = total
         self.n_layers = n_layers
