@@ -65,9 +65,12 @@ def _close(got, ref, what):
     assert np.all(err <= bound), f"{what}: coverage off by {np.max(err / bound):.3g} x bound"
 
 
-@pytest.mark.parametrize("name", ["qwen7b-1layer", "ragged-small", "d64-bf16"])
+@pytest.mark.parametrize("name", ["qwen7b-1layer", "ragged-small", "d64-bf16", "tiny-f32"])
 def test_coverage_matches_oracle(name):
-    wl = {"qwen7b-1layer": QWEN1, "ragged-small": RAGGED, "d64-bf16": D64}[name]
+    """bf16 cases run the tensor-core scoring kernels, the fp32 case the
+    CUDA-core ones."""
+    wl = {"qwen7b-1layer": QWEN1, "ragged-small": RAGGED, "d64-bf16": D64,
+          "tiny-f32": S.WORKLOADS["tiny-f32"]}[name]
     n_dec = 16
     li = S.make_layer(wl, 0)
     dec = S.make_decode_queries(wl, 0, li, n_dec)
