@@ -12,6 +12,16 @@
  *   5. keep the last token plus the top C-1 keys (Section 3.2.3);
  *   6. gather the kept K/V rows, in temporal order, into a compact cache
  *      (Appendix B).
+ * Beyond the window-statistics path (mmshift_select and its steps):
+ *   - proxy statistics over every prompt query (mmshift_prefill_stats,
+ *     mmshift_select_with_stats) or over the prefill hidden states, with the
+ *     proxies sampled in hidden space and projected by W_Q on the tensor
+ *     cores (mmshift_hidden_stats, mmshift_build_hidden_proxies), as
+ *     Section 3.2.1 writes them;
+ *   - a budget per layer and KV head (mmshift_select_head_budgets,
+ *     mmshift_topk_head_budgets; Section 3.1's C_{l,h});
+ *   - the attention-mass coverage of a kept set for given decode queries
+ *     (mmshift_coverage; Section 1, Fig. 1b).
  *
  * Conventions shared by every entry point:
  *   - All pointers except the ones marked "host" are device pointers. The
