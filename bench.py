@@ -575,21 +575,22 @@ def run_gpu(args, wl):
 
     hb_dev = torch.from_numpy(hb_host).to(dev) if hb_host is not None else None
 
-    def select(Kx, Vx, Qx, Xx, dbg=None, sev=None):
+    def select(Kx, Vx, Qx, Xx, dbg=None, sev=None, outs=None):
+        oi, ok, ov = outs if outs is not None else (out_idx, out_k, out_v)
         if hb_dev is not None:
-            M.check(M.mmshift_select_head_budgets(shape, Kx, Vx, Qx, None, hb_dev, params, out_idx,
-                                                  None, out_k, out_v, dbg, ws, ws_bytes, stream),
+            M.check(M.mmshift_select_head_budgets(shape, Kx, Vx, Qx, None, hb_dev, params, oi,
+                                                  None, ok, ov, dbg, ws, ws_bytes, stream),
                     "mmshift_select_head_budgets")
         elif pre is None:
-            M.check(M.mmshift_select(shape, Kx, Vx, Qx, None, params, out_idx, out_k, out_v, dbg,
+            M.check(M.mmshift_select(shape, Kx, Vx, Qx, None, params, oi, ok, ov, dbg,
                                      ws, ws_bytes, stream), "mmshift_select")
         elif pre.kind == "prefill":
             st = pre.run(Xx, stream, sev)
-            M.check(M.mmshift_select_with_stats(shape, Kx, Vx, Qx, st, params, out_idx, out_k, out_v,
+            M.check(M.mmshift_select_with_stats(shape, Kx, Vx, Qx, st, params, oi, ok, ov,
                                                 dbg, ws, ws_bytes, stream), "mmshift_select_with_stats")
         else:
             px = pre.run(Xx, stream, sev)
-            M.check(M.mmshift_select(shape, Kx, Vx, Qx, px, params, out_idx, out_k, out_v, dbg,
+            M.check(M.mmshift_select(shape, Kx, Vx, Qx, px, params, oi, ok, ov, dbg,
                                      ws, ws_bytes, stream), "mmshift_select")
 
     def step(dbg=None, sev=None):
@@ -636,10 +637,15 @@ def run_gpu(args, wl):
     ov_h = torch.empty_like(ok_h, pin_memory=True)
     e_steps = max(1, args.steps)
     # Every step copies its inputs from pinned host memory and reads its
-    # results back. The inputs are double-buffered on the device, so the
-    # copies of step k+1 (on a copy stream) overlap the selection of step k;
-    # a buffer is refilled only after the selection that read it.
-    Kb, Vb, Qb = [K, torch.empty_like(K)], [V, torch.empty_like(V)], [Q, torch.empty_like(Q)]
+    # results back. K, Qwin (and the prompt queries / hidden states of
+    # --stats) are double-buffered on the device, so their copies for step
+    # k+1 (on a copy stream) overlap the selection of step k; a buffer is
+    # refilled only after the selection that read it. V stays in pinned host
+    # memory: the gather reads only the kept rows across the host link. The
+    # outputs are double-buffered too and copied back on the copy stream.
+    Kb, Qb = [K, torch.empty_like(K)], [Q, torch.empty_like(Q)]
+    outs = [(out_idx, out_k, out_v),
+            (torch.empty_like(out_idx), torch.empty_like(out_k), torch.empty_like(out_v))]
     if pre:
         X_pin = torch.empty(pre.x.shape, dtype=pre.x.dtype, pin_memory=True)
         X_pin.copy_(pre.x)
@@ -647,12 +653,13 @@ def run_gpu(args, wl):
     cstream = torch.cuda.Stream(dev)
     ready = [torch.cuda.Event() for _ in range(2)]
     free = [torch.cuda.Event() for _ in range(2)]
+    done = [torch.cuda.Event() for _ in range(2)]
+    drained = [torch.cuda.Event() for _ in range(2)]
 
     def copy_in(i):
         cstream.wait_event(free[i])
         with torch.cuda.stream(cstream):
             Kb[i].copy_(K_pin, non_blocking=True)
-            Vb[i].copy_(V_pin, non_blocking=True)
             Qb[i].copy_(Q_pin, non_blocking=True)
             if pre:
                 Xb[i].copy_(X_pin, non_blocking=True)
@@ -660,20 +667,29 @@ def run_gpu(args, wl):
 
     def select_out(i):
         stream.wait_event(ready[i])
-        select(Kb[i], Vb[i], Qb[i], Xb[i] if pre else None)
+        stream.wait_event(drained[i])
+        select(Kb[i], V_pin, Qb[i], Xb[i] if pre else None, outs=outs[i])
         free[i].record(stream)
-        idx_h.copy_(out_idx, non_blocking=True)
-        ok_h.copy_(out_k, non_blocking=True)
-        ov_h.copy_(out_v, non_blocking=True)
+        done[i].record(stream)
+
+    def copy_out(i):
+        cstream.wait_event(done[i])
+        with torch.cuda.stream(cstream):
+            idx_h.copy_(outs[i][0], non_blocking=True)
+            ok_h.copy_(outs[i][1], non_blocking=True)
+            ov_h.copy_(outs[i][2], non_blocking=True)
+        drained[i].record(cstream)
 
     def e2e(nsteps):
-        for ev in free:
+        for ev in free + drained:
             ev.record(stream)
         copy_in(0)
         for k in range(nsteps):
             if k + 1 < nsteps:
                 copy_in((k + 1) % 2)
             select_out(k % 2)
+            copy_out(k % 2)
+        stream.wait_stream(cstream)     # the last results are on the host
 
     e2e(2)                        # untimed warm-up of the pinned host buffers and streams
     torch.cuda.synchronize()
@@ -684,7 +700,10 @@ def run_gpu(args, wl):
     e1.record(stream)
     torch.cuda.synchronize()
     e_ms = ranks.max(e0.elapsed_time(e1) / e_steps, dev)
-    h2d = sum(t.numel() * t.element_size() for t in (K_pin, V_pin, Q_pin))
+    # K, Qwin (and X) copied, plus the kept V rows the gather reads from host memory
+    kept_rows = int(out_idx.numel())
+    h2d = sum(t.numel() * t.element_size() for t in (K_pin, Q_pin)) + kept_rows * wl.head_dim * \
+        V_pin.element_size()
     if pre:
         h2d += X_pin.numel() * X_pin.element_size()
     d2h = sum(t.numel() * t.element_size() for t in (idx_h, ok_h, ov_h))
@@ -779,8 +798,10 @@ def run_gpu(args, wl):
         **extra_roofs,
         "cpu_baseline": cpu,
         "e2e": {"value": job_value(T * L, world, e_ms), "unit": UNIT, "ms_per_step": e_ms,
-                "pipeline": "inputs double-buffered on the device: the host-to-device copies "
-                            "of step k+1 overlap the selection of step k",
+                "pipeline": "K and Qwin double-buffered on the device (copies of step k+1 overlap "
+                            "the selection of step k); V read in place from pinned host memory, "
+                            "only the kept rows, by the gather; outputs double-buffered and "
+                            "copied back on the copy stream",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "clocks": clk,
         "gpu_launches": launches,

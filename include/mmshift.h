@@ -26,7 +26,14 @@
  * Conventions shared by every entry point:
  *   - All pointers except the ones marked "host" are device pointers. The
  *     caller owns every buffer; the library allocates no device memory and,
- *     apart from mmshift_poll_status, never synchronises.
+ *     apart from mmshift_poll_status, never synchronises. One exception:
+ *     V, of which only the kept rows are read (by the gather), may also be
+ *     page-locked host memory mapped into the device's address space at the
+ *     same address (cudaHostAlloc / cudaHostRegister memory under unified
+ *     addressing); the gather then reads just those rows across the
+ *     host link. mmshift_select and mmshift_gather check K, Qwin and V
+ *     with cudaPointerGetAttributes and refuse (MMSHIFT_ERR_INVALID_ARG)
+ *     pageable host memory.
  *   - All work is enqueued on `stream` (a cudaStream_t; NULL is the legacy
  *     default stream) and is asynchronous.
  *   - Host-side validation runs first; on error nothing is enqueued and the

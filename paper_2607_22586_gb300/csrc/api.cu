@@ -258,6 +258,27 @@ static mmshift_status stats_job(const mmshift_shape* s, int64_t qfull_layer_stri
   return MMSHIFT_OK;
 }
 
+// Whether kernels may read `p` with plain loads: device or managed memory,
+// or page-locked host memory mapped at the same address (unified
+// addressing). Pageable host memory is refused.
+static bool device_readable(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();   // clear the sticky error of a failed query
+    return false;
+  }
+  if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) return true;
+  return a.type == cudaMemoryTypeHost && a.devicePointer == p;
+}
+static bool device_memory(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+}
+
 // The hidden-space proxy job of a call: shapes, tiles and RoPE positions.
 static mmshift_status hidden_job(const mmshift_shape* s, int32_t d_model, const mmshift_params* p,
                                  const int32_t* rope_pos, HiddenJob* J) {
@@ -307,6 +328,10 @@ static mmshift_status select_impl(const mmshift_shape* s, const void* K, const v
   P.part_slots = P.use_umma ? kUmmaPartSlots : 1;
   Buffers bf;
   if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
+  // K and Qwin are streamed by every pass: device memory; V is read only for
+  // the kept rows and may also be mapped page-locked host memory
+  if (!device_memory(K) || !device_memory(Qwin) || !device_readable(V))
+    return MMSHIFT_ERR_INVALID_ARG;
   bf.proxies_in = proxies_in;
   bf.stats_in = stats_in;
   bf.head_budget = head_budgets;
@@ -578,6 +603,7 @@ mmshift_status mmshift_gather(const mmshift_shape* s, const void* K, const void*
   if (!K || !V || !idx || !out_K || !out_V) return MMSHIFT_ERR_INVALID_ARG;
   Buffers bf;
   if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
+  if (!device_readable(K) || !device_readable(V)) return MMSHIFT_ERR_INVALID_ARG;
   const cudaError_t e = launch_gather(P, bf, (cudaStream_t)stream, K, V, idx, out_K, out_V);
   return e == cudaSuccess ? MMSHIFT_OK : cuda_fail(e);
 }

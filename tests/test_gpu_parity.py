@@ -6,6 +6,7 @@ import pytest
 import torch
 
 import paper_2607_22586_gb300 as M
+from paper_2607_22586_gb300 import _lib as LB
 from paper_2607_22586_gb300 import synth as S
 from oracle import mmshift_oracle as O
 from tests import parity as PT
@@ -250,3 +251,35 @@ def test_gather_bit_exact_and_bad_index_reported():
     assert M.mmshift_poll_status(ws) == M._lib.MMSHIFT_ERR_DEVICE
     assert torch.all(ok_t[0, 0, 0] == 0)
     assert M.mmshift_poll_status(ws) == 0
+
+
+def test_values_in_mapped_host_memory():
+    """V may live in page-locked host memory (only the kept rows are read):
+    the results equal those with V on the device; pageable host memory for V,
+    and host memory for K, are refused before anything is launched."""
+    wl = RAGGED
+    li = S.make_layer(wl, 0)
+    h = PT.hyper(n_proxies=64, n_groups=4, seed=12)
+    ref = PT.gpu_select(wl, [li], h)
+    shape = PT.shape_of(wl)
+    params = PT.abi_params(h)
+    rows = M.mmshift_output_rows(shape)
+    ws_bytes = M.mmshift_workspace_size(shape, params)
+    ws = torch.zeros(ws_bytes, dtype=torch.uint8, device="cuda")
+    K, Q = PT.dev(li.K[None], wl.dtype), PT.dev(li.Qwin[None], wl.dtype)
+    V_dev = PT.dev(li.V[None], wl.dtype)
+    V_pin = V_dev.cpu().pin_memory()
+    idx = torch.full((1, rows, wl.n_kv_heads), -7, dtype=torch.int32, device="cuda")
+    ok = torch.empty((1, rows, wl.n_kv_heads, wl.head_dim), dtype=torch.bfloat16, device="cuda")
+    ov = torch.empty_like(ok)
+    M.check(M.mmshift_select(shape, K, V_pin, Q, None, params, idx, ok, ov, None, ws, ws_bytes),
+            "select with pinned V")
+    assert M.mmshift_poll_status(ws) == 0
+    np.testing.assert_array_equal(PT.host(idx), ref["idx"])
+    np.testing.assert_array_equal(PT.host(ok), ref["out_k"])
+    np.testing.assert_array_equal(PT.host(ov), ref["out_v"])
+    V_pageable = V_dev.cpu()
+    assert M.mmshift_select(shape, K, V_pageable, Q, None, params, idx, ok, ov, None, ws,
+                            ws_bytes) == LB.MMSHIFT_ERR_INVALID_ARG
+    assert M.mmshift_select(shape, K.cpu().pin_memory(), V_dev, Q, None, params, idx, ok, ov, None,
+                            ws, ws_bytes) == LB.MMSHIFT_ERR_INVALID_ARG
