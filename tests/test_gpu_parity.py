@@ -283,3 +283,44 @@ def test_values_in_mapped_host_memory():
                             ws_bytes) == LB.MMSHIFT_ERR_INVALID_ARG
     assert M.mmshift_select(shape, K.cpu().pin_memory(), V_dev, Q, None, params, idx, ok, ov, None,
                             ws, ws_bytes) == LB.MMSHIFT_ERR_INVALID_ARG
+
+
+def test_select_captured_in_a_cuda_graph():
+    """mmshift_select enqueues only stream work (tensor maps are encoded on
+    the host), so a serving loop can capture it once in a CUDA graph and
+    replay it: the replay gives the same results as a direct call."""
+    wl = RAGGED.replace(seq_lens=(3000, 1333), n_visual=(2990, 1300), budgets=(256, 64), n_layers=2)
+    lis = [S.make_layer(wl, l) for l in range(2)]
+    h = PT.hyper(n_proxies=64, n_groups=4, seed=6)
+    ref = PT.gpu_select(wl, lis, h)
+    shape = PT.shape_of(wl, 2)
+    params = PT.abi_params(h)
+    rows = M.mmshift_output_rows(shape)
+    ws_bytes = M.mmshift_workspace_size(shape, params)
+    ws = torch.zeros(ws_bytes, dtype=torch.uint8, device="cuda")
+    K = PT.dev(np.stack([li.K for li in lis]), wl.dtype)
+    V = PT.dev(np.stack([li.V for li in lis]), wl.dtype)
+    Q = PT.dev(np.stack([li.Qwin for li in lis]), wl.dtype)
+    idx = torch.full((2, rows, wl.n_kv_heads), -7, dtype=torch.int32, device="cuda")
+    ok = torch.zeros((2, rows, wl.n_kv_heads, wl.head_dim), dtype=torch.bfloat16, device="cuda")
+    ov = torch.zeros_like(ok)
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):      # one call outside the capture (module loading, attributes)
+        M.check(M.mmshift_select(shape, K, V, Q, None, params, idx, ok, ov, None, ws, ws_bytes, side),
+                "warm-up")
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    idx.fill_(-7)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        st = torch.cuda.current_stream()
+        M.check(M.mmshift_select(shape, K, V, Q, None, params, idx, ok, ov, None, ws, ws_bytes, st),
+                "captured select")
+    for _ in range(2):
+        idx.fill_(-7)
+        g.replay()
+    torch.cuda.synchronize()
+    assert M.mmshift_poll_status(ws) == 0
+    np.testing.assert_array_equal(PT.host(idx), ref["idx"])
+    np.testing.assert_array_equal(PT.host(ok), ref["out_k"])
