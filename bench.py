@@ -63,9 +63,9 @@ SFU_EX2_PER_SM_CLK = 32          # MUFU.EX2 lanes per SM per clock on GB300 (mea
 # launch-list pass with the two DRAM byte counters), mean over the five
 # device-resident steps. It describes only the score_umma.cu it was measured
 # on (checked by hash).
-SCORE_TRAFFIC = {"source_sha256_16": "08cd22d64d3ad96f", "workload": "qwen7b-28l-32k",
-                 "proxies": "paper", "softmax_pass": 1502.5e6 + 420.8e6,
-                 "mass_pass": 1699.8e6 + 479.7e6}
+SCORE_TRAFFIC = {"source_sha256_16": "8695137d6647c765", "workload": "qwen7b-28l-32k",
+                 "proxies": "paper", "softmax_pass": 1502.7e6 + 420.9e6,
+                 "mass_pass": 1801.5e6 + 480.5e6}
 # DRAM traffic of the prompt-query statistics pass (both kernels) per launch
 # of the default workload, from one ncu capture of a 4-layer slice scaled by 7
 # (partial kernel 939.590912 MB read + 3.059712 MB written, merge 11.026176 MB

@@ -10,8 +10,11 @@
 // block). Teams of one CTA (softmax: one CTA pair) per proxy block walk
 // contiguous ranges of key splits, so the team reads each K tile together
 // (DRAM once, then L2) and a stationary block changes only with the (layer,
-// request, head). The split boundaries (and so the merge order of the
-// softmax partials) are those of the CUDA-core path.
+// request, head). Where the SMs are not a multiple of the blocks, the teams
+// take a little less and the CTAs left over share the teams' remaining
+// splits block by block (work lists, below), so no SM idles. The split
+// boundaries (and so the merge order of the softmax partials) are those of
+// the CUDA-core path.
 //
 // Softmax pass (softmax_pair_kernel): CTA pairs and 2-SM MMAs, below. The
 //   accumulator lane is a proxy row, so each thread keeps its row's running
@@ -31,10 +34,13 @@
 // stops issuing work and still frees its TMEM.
 #include <cudaTypedefs.h>
 
+#include <algorithm>
+#include <cmath>
 #include <mutex>
 
 #include "common.cuh"
 #include "umma.cuh"
+#include "work_lists.h"
 
 namespace mmshift {
 namespace {
@@ -57,7 +63,52 @@ struct Sched {
   int32_t gpt;                           // mass pass: groups per regular block
   int32_t n_reg;                         // mass pass: regular blocks
   int32_t anchor_merged;                 // mass pass: anchor rows ride on the last block
+  // per-worker lists (work_lists.h); a worker is a CTA (mass pass) or a CTA
+  // pair (softmax pass)
+  WorkLists wl;
 };
+
+// A worker's walk over its list, one split row at a time. The plain team
+// schedule is resolved once: a = the worker's first split row, c = its
+// block. A list is followed segment by segment: c = current segment, a =
+// split rows of the worker before it. LISTS (a template argument of both
+// kernels) selects the list form at compile time, so the plain-team kernels
+// carry no list walk.
+struct Walk {
+  int n;      // split rows of the worker
+  int a, c;
+};
+
+template <bool LISTS>
+__device__ __forceinline__ Walk walk_begin(const Sched& S, int w, int nw) {
+  Walk k;
+  if (LISTS) {
+    k.n = 0;
+    for (int i = 0; i < S.wl.nseg[w]; ++i) k.n += S.wl.seg[w][i].e - (S.wl.seg[w][i].bt >> 8);
+    k.a = 0;
+    k.c = 0;
+  } else {
+    const int nteams = nw / S.ntiles, team = w / S.ntiles;
+    const int rows = S.units / S.ntiles;
+    k.a = (int)((long long)team * rows / nteams);
+    k.n = (int)((long long)(team + 1) * rows / nteams) - k.a;
+    k.c = w % S.ntiles;
+  }
+  return k;
+}
+
+// Unit index of the worker's i-th split row; i grows by one per call.
+template <bool LISTS>
+__device__ __forceinline__ int walk_unit(const Sched& S, int w, Walk& k, int i) {
+  if (!LISTS) return (k.a + i) * S.ntiles + k.c;
+  for (;;) {
+    const PackedSeg p = S.wl.seg[w][k.c];
+    const int b = p.bt >> 8, len = p.e - b;
+    if (i - k.a < len) return (b + i - k.a) * S.ntiles + (p.bt & 255);
+    k.a += len;
+    ++k.c;
+  }
+}
 
 struct Unit {
   int l, b, h, tile, split, t0, t1;
@@ -247,7 +298,7 @@ __device__ __forceinline__ float group_sum(uint32_t tcol, const float* nc, int n
   return (a0 + a1) + (a2 + a3);
 }
 
-template <int D>
+template <int D, bool LISTS>
 __global__ void __launch_bounds__(NTHREADS, 1)
     mass_umma_kernel(const __grid_constant__ CUtensorMap kmap,
                       const __grid_constant__ CUtensorMap pmap, const __grid_constant__ Problem P,
@@ -265,17 +316,13 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   volatile int* abort_ = &abort_flag;
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  // Team schedule: the grid is a multiple of the stationary blocks per
-  // (request, KV head); team j = CTAs [j*ntiles, (j+1)*ntiles), one per block.
-  // A team walks a contiguous range of key splits (over layers, requests and
-  // heads); all its CTAs read the same split at the same time, so each K tile
-  // comes from DRAM once and from L2 for the others, and a CTA reloads its
-  // stationary block only when the (layer, request, head) changes.
-  const int nteams = gridDim.x / S.ntiles;
-  const int team = blockIdx.x / S.ntiles, my_tile = blockIdx.x % S.ntiles;
-  const int nsplit_rows = S.units / S.ntiles;
-  const int s_begin = (int)((long long)team * nsplit_rows / nteams);
-  const int s_end = (int)((long long)(team + 1) * nsplit_rows / nteams);
+  // Work list of this CTA (Sched). In a team (one CTA per stationary block)
+  // all CTAs walk the same key splits (over layers, requests and heads) at the
+  // same time, so each K tile comes from DRAM once and from L2 for the others;
+  // a CTA reloads its stationary block only when the (layer, request, head)
+  // or the block changes. The three roles walk the same list.
+  const int wk = blockIdx.x;
+  Walk walk = walk_begin<LISTS>(S, wk, gridDim.x);
 
   if (threadIdx.x == 0) {
     abort_flag = 0;
@@ -308,12 +355,13 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       int stage = 0;
       uint32_t phase = 0, sphase = 0;
       long long prev = -1;
-      for (int sr = s_begin; sr < s_end; ++sr) {
-        const int u = sr * S.ntiles + my_tile;
+      bool ok = true;
+      for (int i = 0; i < walk.n && ok; ++i) {
+        const int u = walk_unit<LISTS>(S, wk, walk, i);
         const Unit x = decode(P, S, u);
         const long long key = block_key(P, S, x);
         if (key != prev) {
-          if (!mbar_wait(&sempty, sphase ^ 1u, abort_)) break;
+          if (!mbar_wait(&sempty, sphase ^ 1u, abort_)) { ok = false; break; }
           const Block k = mass_block(P, S, x.tile);
           const int row0 = k.row0, rows = k.rows;
           mbar_expect_tx(&sfull, (uint32_t)(rows * D * 2));
@@ -325,7 +373,6 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           prev = key;
         }
         const int kbase = P.req[x.b].tok_off;
-        bool ok = true;
         for (int kt = x.t0; kt < x.t1; kt += BK) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_)) { ok = false; break; }
           mbar_expect_tx(&full[stage], (uint32_t)SM::STAGE_BYTES);
@@ -334,7 +381,6 @@ __global__ void __launch_bounds__(NTHREADS, 1)
                         x.h * D + c * 64, kbase + kt, x.l);
           if (++stage == NSTAGE) { stage = 0; phase ^= 1u; }
         }
-        if (!ok) break;
       }
     }
   } else if (warp == 1) {
@@ -344,19 +390,19 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       uint32_t phase = 0, bphase = 0, sphase = 0;   // bphase: one phase bit per accumulator
       long long prev = -1;
       uint32_t idesc = 0;
-      for (int sr = s_begin; sr < s_end; ++sr) {
-        const int u = sr * S.ntiles + my_tile;
+      bool ok = true;
+      for (int i = 0; i < walk.n && ok; ++i) {
+        const int u = walk_unit<LISTS>(S, wk, walk, i);
         const Unit x = decode(P, S, u);
         const long long key = block_key(P, S, x);
         if (key != prev) {
           if (prev != -1) mma_commit(&sempty);   // old block free once its MMAs finish
-          if (!mbar_wait(&sfull, sphase, abort_)) break;
+          if (!mbar_wait(&sfull, sphase, abort_)) { ok = false; break; }
           sphase ^= 1u;
           fence_after();
           idesc = idesc_bf16_f32(128, mass_block(P, S, x.tile).rows);
           prev = key;
         }
-        bool ok = true;
         // accumulator = parity of the tile's index within its split, so a
         // split's tiles reach the same epilogue warpgroups whatever ran before
         for (int kt = x.t0, j = 0; kt < x.t1; kt += BK, ++j) {
@@ -379,7 +425,6 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           if (++stage == NSTAGE) { stage = 0; phase ^= 1u; }
           bphase ^= 1u << buf;
         }
-        if (!ok) break;
       }
     }
   } else {
@@ -396,8 +441,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     const float alpha = P.alpha;
     uint32_t bphase = 0;                  // one phase bit per accumulator
     long long prev_blk = -1;
-    for (int sr = s_begin; sr < s_end; ++sr) {
-      const int u = sr * S.ntiles + my_tile;
+    bool ok = true;
+    for (int i = 0; i < walk.n && ok; ++i) {
+      const int u = walk_unit<LISTS>(S, wk, walk, i);
       const Unit x = decode(P, S, u);
       const ReqInfo R = P.req[x.b];
       const long long key = block_key(P, S, x);
@@ -410,7 +456,6 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         __syncwarp();
         prev_blk = key;
       }
-      bool ok = true;
       for (int kt = x.t0, j = 0; kt < x.t1; kt += BK, ++j) {
         const int buf = j & 1;
         if (buf != par) continue;
@@ -439,7 +484,6 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         fence_before();
         mbar_arrive(&tempty[buf]);
       }
-      if (!ok) break;
     }
   }
 
@@ -476,7 +520,7 @@ struct PairSmem {
   static constexpr int DYN_BYTES = 1024 + STAT_BYTES + RING_BYTES;
 };
 
-template <int D>
+template <int D, bool LISTS>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
     softmax_pair_kernel(const __grid_constant__ CUtensorMap kmap,
                         const __grid_constant__ CUtensorMap pmap, const __grid_constant__ Problem P,
@@ -496,13 +540,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const uint32_t rank = cluster_rank();
-  // team schedule as in the one-SM kernel, counted in pairs
-  const int pair = blockIdx.x >> 1;
-  const int nteams = (gridDim.x >> 1) / S.ntiles;
-  const int team = pair / S.ntiles, my_tile = pair % S.ntiles;
-  const int nsplit_rows = S.units / S.ntiles;
-  const int s_begin = (int)((long long)team * nsplit_rows / nteams);
-  const int s_end = (int)((long long)(team + 1) * nsplit_rows / nteams);
+  // work lists as in the one-SM kernel, one per pair
+  const int wk = blockIdx.x >> 1;
+  Walk walk = walk_begin<LISTS>(S, wk, gridDim.x >> 1);
 
   if (threadIdx.x == 0) {
     abort_flag = 0;
@@ -536,11 +576,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
       int stage = 0;
       uint32_t phase = 0, sphase = 0;
       long long prev = -1;
-      for (int sr = s_begin; sr < s_end; ++sr) {
-        const Unit x = decode(P, S, sr * S.ntiles + my_tile);
+      bool ok = true;
+      for (int i = 0; i < walk.n && ok; ++i) {
+        const Unit x = decode(P, S, walk_unit<LISTS>(S, wk, walk, i));
         const long long key = block_key(P, S, x);
         if (key != prev) {
-          if (!mbar_wait(&sempty, sphase ^ 1u, abort_)) break;
+          if (!mbar_wait(&sempty, sphase ^ 1u, abort_)) { ok = false; break; }
           if (rank == 0) mbar_expect_tx(&sfull, (uint32_t)(2 * PROWS * D * 2));
           const uint32_t bar = mapa(smem_u32(&sfull), 0);
           const int zc = (x.l * P.B + x.b) * P.Hkv + x.h;
@@ -552,7 +593,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
           prev = key;
         }
         const int kbase = P.req[x.b].tok_off + (int)rank * (PBK / 2);
-        bool ok = true;
         for (int kt = x.t0; kt < x.t1; kt += PBK) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_)) { ok = false; break; }
           if (rank == 0) mbar_expect_tx(&full[stage], (uint32_t)(2 * SM::STAGE_BYTES));
@@ -562,7 +602,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
                              x.h * D + c * 64, kbase + kt, x.l);
           if (++stage == PNSTAGE) { stage = 0; phase ^= 1u; }
         }
-        if (!ok) break;
       }
     }
   } else if (warp == 1) {
@@ -572,17 +611,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
       uint32_t phase = 0, bphase = 0, sphase = 0;
       long long prev = -1;
       const uint32_t idesc = idesc_bf16_f32(2 * PROWS, PBK);
-      for (int sr = s_begin; sr < s_end; ++sr) {
-        const Unit x = decode(P, S, sr * S.ntiles + my_tile);
+      bool ok = true;
+      for (int i = 0; i < walk.n && ok; ++i) {
+        const Unit x = decode(P, S, walk_unit<LISTS>(S, wk, walk, i));
         const long long key = block_key(P, S, x);
         if (key != prev) {
           if (prev != -1) mma_commit_pair(&sempty, 0x3);   // old block free once its MMAs finish
-          if (!mbar_wait(&sfull, sphase, abort_)) break;
+          if (!mbar_wait(&sfull, sphase, abort_)) { ok = false; break; }
           sphase ^= 1u;
           fence_after();
           prev = key;
         }
-        bool ok = true;
         for (int kt = x.t0, j = 0; kt < x.t1; kt += PBK, ++j) {
           const int buf = j & 1;
           if (!mbar_wait(&full[stage], phase, abort_) ||
@@ -603,7 +642,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
           if (++stage == PNSTAGE) { stage = 0; phase ^= 1u; }
           bphase ^= 1u << buf;
         }
-        if (!ok) break;
       }
     }
   } else {
@@ -616,14 +654,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
     const int c_lo = wg * (PBK / 4);
     const uint32_t tempty_lead[2] = {mapa(smem_u32(&tempty[0]), 0), mapa(smem_u32(&tempty[1]), 0)};
     uint32_t bphase = 0;
-    for (int sr = s_begin; sr < s_end; ++sr) {
-      const Unit x = decode(P, S, sr * S.ntiles + my_tile);
+    bool ok = true;
+    for (int i = 0; i < walk.n && ok; ++i) {
+      const Unit x = decode(P, S, walk_unit<LISTS>(S, wk, walk, i));
       const ReqInfo R = P.req[x.b];
       // (reference max, sum of exp2(x - max)) of this thread's row over its
       // quarter of every tile of the split, restarted per split
       float m_run = -INFINITY, z_run = 0.f;
       bool first = true;
-      bool ok = true;
       for (int kt = x.t0, j = 0; kt < x.t1; kt += PBK, ++j) {
         const int buf = j & 1;
         const uint32_t ph = (bphase >> buf) & 1u;
@@ -709,6 +747,10 @@ int sm_count() {
   return n;
 }
 
+// the scoring kernels take two tensor maps, Problem, Sched and Buffers by value
+static_assert(2 * sizeof(CUtensorMap) + sizeof(Problem) + sizeof(Sched) + sizeof(Buffers) <= 32764,
+              "kernel parameters above the 32,764-byte limit");
+
 template <int D>
 cudaError_t launch_d(const Problem& P, const Buffers& bf, cudaStream_t st, const void* K,
                      cudaEvent_t* ev) {
@@ -724,33 +766,41 @@ cudaError_t launch_d(const Problem& P, const Buffers& bf, cudaStream_t st, const
   const int nsm = sm_count();
   if (nsm <= 0) return cudaErrorInvalidDevice;
   cudaError_t e;
-  if ((e = cudaFuncSetAttribute(softmax_pair_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                PairSmem<D>::DYN_BYTES)) != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(mass_umma_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                SM::DYN_BYTES)) != cudaSuccess) return e;
-  const Sched s1 = make_sched(P, 1), s2 = make_sched(P, 2);
-  // whole teams of ntiles CTAs (one per stationary block), at most one CTA
-  // per SM while the work allows
-  auto grid_of = [nsm](const Sched& s) {
-    const int rows = s.units / s.ntiles;
-    const int nteams = std::max(1, std::min(nsm / s.ntiles, rows));
-    return nteams * s.ntiles;
-  };
+  for (auto f : {softmax_pair_kernel<D, false>, softmax_pair_kernel<D, true>})
+    if ((e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  PairSmem<D>::DYN_BYTES)) != cudaSuccess) return e;
+  for (auto f : {mass_umma_kernel<D, false>, mass_umma_kernel<D, true>})
+    if ((e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  SM::DYN_BYTES)) != cudaSuccess) return e;
+  Sched s1 = make_sched(P, 1), s2 = make_sched(P, 2);
   if (ev && (e = cudaEventRecord(ev[1], st)) != cudaSuccess) return e;
   if (s1.units) {
-    // pairs of CTAs (clusters of two), whole teams of ntiles pairs
-    const int rows = s1.units / s1.ntiles;
-    const int nteams = std::max(1, std::min(nsm / (2 * s1.ntiles), rows));
-    softmax_pair_kernel<D><<<2 * nteams * s1.ntiles, NTHREADS, PairSmem<D>::DYN_BYTES, st>>>(
-        kmap, pmap, P, s1, bf);
+    // softmax pass: workers are CTA pairs (clusters of two), one per two SMs
+    const int pairs = nsm / 2;
+    if (balance_workers(s1.wl, s1.ntiles, s1.units / s1.ntiles, pairs)) {
+      softmax_pair_kernel<D, true><<<2 * pairs, NTHREADS, PairSmem<D>::DYN_BYTES, st>>>(
+          kmap, pmap, P, s1, bf);
+    } else {
+      // whole teams of ntiles pairs
+      const int rows = s1.units / s1.ntiles;
+      const int grid_pairs = std::max(1, std::min(pairs / s1.ntiles, rows)) * s1.ntiles;
+      softmax_pair_kernel<D, false><<<2 * grid_pairs, NTHREADS, PairSmem<D>::DYN_BYTES, st>>>(
+          kmap, pmap, P, s1, bf);
+    }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   if (ev && (e = cudaEventRecord(ev[2], st)) != cudaSuccess) return e;
   if ((e = launch_merge(P, bf, st)) != cudaSuccess) return e;
   if (ev && (e = cudaEventRecord(ev[3], st)) != cudaSuccess) return e;
   if (s2.units) {
-    mass_umma_kernel<D><<<grid_of(s2), NTHREADS, SM::DYN_BYTES, st>>>(kmap, pmap, P,
-                                                                                      s2, bf);
+    // mass pass: workers are CTAs, one per SM
+    if (balance_workers(s2.wl, s2.ntiles, s2.units / s2.ntiles, nsm)) {
+      mass_umma_kernel<D, true><<<nsm, NTHREADS, SM::DYN_BYTES, st>>>(kmap, pmap, P, s2, bf);
+    } else {
+      const int rows = s2.units / s2.ntiles;
+      const int grid = std::max(1, std::min(nsm / s2.ntiles, rows)) * s2.ntiles;
+      mass_umma_kernel<D, false><<<grid, NTHREADS, SM::DYN_BYTES, st>>>(kmap, pmap, P, s2, bf);
+    }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   return cudaSuccess;
