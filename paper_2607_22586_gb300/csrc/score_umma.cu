@@ -60,9 +60,7 @@ struct Sched {
   int32_t uoff[MMSHIFT_MAX_BATCH + 1];  // per-layer units, prefix over requests
   int32_t ntiles;                        // stationary blocks per (request, KV head)
   int32_t units;                         // total units of the launch
-  int32_t gpt;                           // mass pass: groups per regular block
-  int32_t n_reg;                         // mass pass: regular blocks
-  int32_t anchor_merged;                 // mass pass: anchor rows ride on the last block
+  int32_t last_groups;                   // mass pass: groups of the last block (see mass_block)
   // per-worker lists (work_lists.h); a worker is a CTA (mass pass) or a CTA
   // pair (softmax pass)
   WorkLists wl;
@@ -133,27 +131,30 @@ __device__ __forceinline__ Unit decode(const Problem& P, const Sched& S, int u) 
   return x;
 }
 
-// Rows of stationary block t of the mass pass.
+// Rows of stationary block t of the mass pass. Blocks hold whole groups;
+// the last block also holds the anchor rows (they follow the last group's
+// rows in the packed layout) and takes S.last_groups groups, as many as fit
+// beside them; blocks 0 .. ntiles-2 share the other groups as evenly as
+// possible. A group's masses do not depend on the block it lands in.
 struct Block {
   int row0, rows, g0, ng, anchor;
 };
 
 __host__ __device__ inline Block mass_block(const Problem& P, const Sched& S, int t) {
   Block k;
-  if (t < S.n_reg) {
-    k.g0 = t * S.gpt;
-    k.ng = min(P.G - k.g0, S.gpt);
-    k.row0 = k.g0 * P.RG;
-    k.rows = k.ng * P.RG;
-    k.anchor = (S.anchor_merged && t == S.n_reg - 1) ? 1 : 0;
-    if (k.anchor) k.rows += P.anchor_rows;
+  if (t < S.ntiles - 1) {
+    const int nb = S.ntiles - 1, rest = P.G - S.last_groups;
+    const int base = rest / nb, rem = rest % nb;
+    k.ng = base + (t < rem ? 1 : 0);
+    k.g0 = t * base + min(t, rem);
+    k.anchor = 0;
   } else {
-    k.g0 = P.G;
-    k.ng = 0;
-    k.row0 = P.n_group_rows;
-    k.rows = P.anchor_rows;
+    k.g0 = P.G - S.last_groups;
+    k.ng = S.last_groups;
     k.anchor = 1;
   }
+  k.row0 = k.g0 * P.RG;
+  k.rows = k.ng * P.RG + (k.anchor ? P.anchor_rows : 0);
   return k;
 }
 
@@ -724,11 +725,11 @@ Sched make_sched(const Problem& P, int pass) {
   if (pass == 1) {
     s.ntiles = P.Prows_pad / SROWS;
   } else {
-    s.gpt = P.G ? SROWS / P.RG : 1;
-    s.n_reg = P.G ? (P.G + s.gpt - 1) / s.gpt : 0;
-    const int last_rows = P.G ? (P.G - (s.n_reg - 1) * s.gpt) * P.RG : 0;
-    s.anchor_merged = (s.n_reg > 0 && last_rows + P.anchor_rows <= SROWS) ? 1 : 0;
-    s.ntiles = s.n_reg + (s.anchor_merged ? 0 : 1);
+    // fewest blocks of whole groups, the last one with the anchor rows
+    const int per_block = SROWS / P.RG;                      // >= 1 (RG <= SROWS)
+    const int per_last = (SROWS - P.anchor_rows) / P.RG;     // >= 0
+    s.last_groups = min(per_last, P.G);
+    s.ntiles = 1 + (P.G - s.last_groups + per_block - 1) / per_block;
   }
   int acc = 0;
   for (int b = 0; b < P.B; ++b) {
