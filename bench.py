@@ -60,12 +60,12 @@ SFU_EX2_PER_SM_CLK = 32          # MUFU.EX2 lanes per SM per clock on GB300 (mea
 
 # DRAM traffic (read + write) of the two scoring kernels per launch of the
 # default workload: one ncu capture of the full 28-layer workload (the
-# launch-list pass with the two DRAM byte counters), mean over the five
-# device-resident steps. It describes only the score_umma.cu it was measured
-# on (checked by hash).
-SCORE_TRAFFIC = {"source_sha256_16": "8695137d6647c765", "workload": "qwen7b-28l-32k",
-                 "proxies": "paper", "softmax_pass": 1502.7e6 + 420.9e6,
-                 "mass_pass": 1801.5e6 + 480.5e6}
+# launch-list pass with the two DRAM byte counters, first 16 launches), mean
+# over the two steps captured. It describes only the score_umma.cu it was
+# measured on (checked by hash).
+SCORE_TRAFFIC = {"source_sha256_16": "b46d58a266d0a563", "workload": "qwen7b-28l-32k",
+                 "proxies": "paper", "softmax_pass": 1518.0e6 + 420.7e6,
+                 "mass_pass": 1783.9e6 + 479.9e6}
 # DRAM traffic of the prompt-query statistics pass (both kernels) per launch
 # of the default workload, from one ncu capture of a 4-layer slice scaled by 7
 # (partial kernel 939.590912 MB read + 3.059712 MB written, merge 11.026176 MB
