@@ -44,3 +44,14 @@ def test_head_budgets_count_each_heads_kept_rows():
     hb = np.array([[[1, 2, T + 5, 7]]], dtype=np.int32)      # [L][B][Hkv]; one budget above T
     total, k_read, _ = bench.algorithmic(wl, PAPER, hb)
     assert total - k_read == 4 * (1 + 2 + T + 7) * wl.head_dim * 2
+
+
+def test_pyramid_budgets_average_the_uniform_budget():
+    wl = S.WORKLOADS["qwen7b-28l-32k"]
+    hb = bench.pyramid_budgets(wl)
+    C = wl.budgets[0]
+    assert hb.shape == (28, 1, 4) and hb.dtype == np.int32
+    assert hb[0, 0, 0] == round(1.5 * C) and hb[-1, 0, 0] == round(0.5 * C)
+    assert np.all(np.diff(hb[:, 0, 0]) <= 0)                      # shrinking with depth
+    assert abs(hb.mean() - C) <= 1.0                               # C on average
+    assert np.all(hb == hb[:, :, :1])                              # equal across heads
