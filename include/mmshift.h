@@ -142,6 +142,14 @@ typedef struct {
   int32_t launches;   /* out: number of kernels the call enqueued */
   int32_t score_path; /* out: 1 if steps 2-4 ran on the tensor cores (tcgen05),
                          0 if on the CUDA cores (fp32 FMA) */
+  /* Test of the bounded device-side waits; 0 in normal use. Non-zero: on the
+   * tensor-core path, one epilogue warp of the mass pass's first CTA waits
+   * on a barrier that nothing arrives on; after 64 polls (a few ms) it gives
+   * up and aborts its CTA, which waits for the copies and MMAs it already
+   * issued and frees its tensor memory. The call's outputs are then
+   * undefined and mmshift_poll_status returns MMSHIFT_ERR_TIMEOUT; the
+   * context, the workspace and later calls are unaffected. */
+  int32_t test_stuck_wait;
 } mmshift_debug;
 
 #define MMSHIFT_N_STAGES 8
@@ -359,7 +367,10 @@ mmshift_status mmshift_coverage(const mmshift_shape* s, const void* K, const voi
  *    anything is enqueued.
  *  - The first call on a device (with that device current) looks up the
  *    array's device address with cudaGetSymbolAddress; make that first call
- *    before any stream capture on that device.
+ *    before any stream capture on that device. The address is kept for the
+ *    life of the process, so destroying the device's primary context after
+ *    that first call (cudaDeviceReset, which reloads the library's module
+ *    and moves the array) is not supported.
  *  - Every call on a device shares the one array, which keeps the contents of
  *    the last call; nothing in it needs to start at zero (every byte read is
  *    first written by the same call). Calls whose work overlaps on the GPU --

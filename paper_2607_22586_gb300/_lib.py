@@ -72,6 +72,7 @@ class Debug(ctypes.Structure):
         ("mass", ctypes.c_void_p), ("scores", ctypes.c_void_p),
         ("stage_events", ctypes.POINTER(ctypes.c_void_p)), ("n_stage_events", ctypes.c_int32),
         ("launches", ctypes.c_int32), ("score_path", ctypes.c_int32),
+        ("test_stuck_wait", ctypes.c_int32),
     ]
 
 
@@ -364,10 +365,11 @@ def mmshift_poll_status(workspace, stream=None) -> int:
 
 
 def make_debug(proxies=None, group_mass=None, anchor=None, mass=None, scores=None,
-               stage_events=None) -> Debug:
-    """stage_events: sequence of MMSHIFT_N_STAGES + 1 torch.cuda.Event (timing)."""
+               stage_events=None, test_stuck_wait=0) -> Debug:
+    """stage_events: sequence of MMSHIFT_N_STAGES + 1 torch.cuda.Event (timing).
+    test_stuck_wait: test of the bounded device waits (see mmshift.h)."""
     dbg = Debug(proxies=_ptr(proxies), group_mass=_ptr(group_mass), anchor=_ptr(anchor),
-                mass=_ptr(mass), scores=_ptr(scores))
+                mass=_ptr(mass), scores=_ptr(scores), test_stuck_wait=int(test_stuck_wait))
     if stage_events is not None:
         arr = (ctypes.c_void_p * len(stage_events))(*[e.cuda_event for e in stage_events])
         dbg.stage_events = arr

@@ -129,7 +129,7 @@ mmshift_status build_problem(const mmshift_shape* s, const mmshift_params* p, Pr
 }
 
 struct Layout {
-  size_t status, packed, part, cvals, gmass, anchor, bits, scores, total;
+  size_t status, packed, part, cvals, gmass, anchor, bits, scores, refine, refine_stats, total;
 };
 
 Layout layout_of(const Problem& P) {
@@ -145,6 +145,10 @@ Layout layout_of(const Problem& P) {
   w.anchor = o; o += align256(L * P.Hkv * (size_t)P.total_T * sizeof(float));
   w.bits = o;   o += align256(L * P.Hkv * (size_t)P.G * P.total_words * sizeof(uint32_t));
   w.scores = o; o += align256(L * P.Hkv * (size_t)P.total_T * sizeof(float));
+  // count word, the list of proxy elements to recompute in float64, then the
+  // exact window sums they are recomputed from
+  w.refine = o; o += 256 + align256((size_t)proxy_refine_capacity(P) * sizeof(int4));
+  w.refine_stats = o; o += align256(L * P.B * P.Hq * (size_t)5 * P.d * sizeof(float));
   w.total = o;
   return w;
 }
@@ -163,6 +167,10 @@ mmshift_status carve(const Problem& P, void* ws, size_t bytes, Buffers* bf) {
   bf->anchor = reinterpret_cast<float*>(base + w.anchor);
   bf->bits = reinterpret_cast<uint32_t*>(base + w.bits);
   bf->scores = reinterpret_cast<float*>(base + w.scores);
+  bf->refine_count = reinterpret_cast<int*>(base + w.refine);
+  bf->refine_items = reinterpret_cast<int4*>(base + w.refine + 256);
+  bf->refine_cap = (int32_t)proxy_refine_capacity(P);
+  bf->refine_stats = reinterpret_cast<float*>(base + w.refine_stats);
   return MMSHIFT_OK;
 }
 
@@ -200,7 +208,7 @@ int choose_umma(const Problem& P, const void* K) {
 
 // Kernels one mmshift_select call enqueues (reported through mmshift_debug).
 int count_launches(const Problem& P, const Buffers& bf) {
-  int n = 1;                                   // proxies
+  int n = proxy_launches(P, bf);               // proxies (+ float64 refinement)
   n += P.use_umma ? umma_launches(P) : 3;      // softmax pass, merge, mass pass
   if (bf.mass && P.total_T) n += 1;            // mass sum
   if (P.mode == MMSHIFT_SCORE_VOTE && P.G) n += 1;  // coverage vote
@@ -337,6 +345,7 @@ static mmshift_status select_impl(const mmshift_shape* s, const void* K, const v
   bf.head_budget = head_budgets;
   bf.out_count = out_count;
   if (dbg) {
+    P.test_stuck_wait = dbg->test_stuck_wait;
     bf.proxies_out = dbg->proxies;
     if (dbg->group_mass && P.G) bf.gmass = dbg->group_mass;
     if (dbg->anchor) bf.anchor = dbg->anchor;

@@ -52,6 +52,7 @@ struct Problem {
   float rope_theta;
   int32_t rope_off;
   int32_t use_umma;    // steps 2-4 on the tensor cores (set per call)
+  int32_t test_stuck_wait; // test only: see mmshift_debug.test_stuck_wait
   ReqInfo req[MMSHIFT_MAX_BATCH];
 };
 
@@ -72,6 +73,14 @@ struct Buffers {
   const float* stats_in;  // [L][B][2][Hq][d] mean / std of the proxies, or null (window's)
   const int32_t* head_budget; // [L][B][Hkv] budgets C_{l,b,h} in [1, C_b], or null (C_b for all)
   int32_t* out_count;         // [L][B][Hkv] kept rows per head, or null
+  // bf16 proxies whose float32 value lies too close to a rounding boundary
+  // are recomputed in float64 (proxy.cu): the sampler appends them here and a
+  // second kernel redoes them; without a list (null) the sampler redoes them
+  // itself
+  int* refine_count;          // entries appended (may exceed refine_cap)
+  int4* refine_items;         // [refine_cap] (layer * B + request, query head, proxy, dim)
+  float* refine_stats;        // [L][B][Hq][5][d] exact window sums (x0, S1 hi / lo, S2 hi / lo)
+  int32_t refine_cap;
 };
 
 // Whole-prefill statistics job (stats.cu).
@@ -160,6 +169,11 @@ cudaError_t launch_prefill_stats(const StatsJob& J, const void* Q, float* part, 
                                  cudaStream_t st, bool bf16);
 cudaError_t launch_proxy_pack(const Problem& P, const Buffers& bf, cudaStream_t st,
                               const void* qwin);
+// Proxy elements the list of bf holds for a call's shape: at most this many
+// are refined by the second kernel, the rest by the sampler itself.
+int64_t proxy_refine_capacity(const Problem& P);
+// Kernels launch_proxy_pack enqueues for P and bf.
+int proxy_launches(const Problem& P, const Buffers& bf);
 // ev (nullable): stage events 1 (softmax pass), 2 (merge) and 3 (mass pass)
 // are recorded just before the corresponding launch.
 cudaError_t launch_score_simt(const Problem& P, const Buffers& bf, cudaStream_t st,

@@ -102,7 +102,7 @@ __global__ void __launch_bounds__(HTHREADS, 1)
   extern __shared__ unsigned char smraw[];
   unsigned char* sm =
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
-  __shared__ uint64_t full[HSTAGE], empty[HSTAGE], tfull[2], tempty[2];
+  __shared__ uint64_t full[HSTAGE], empty[HSTAGE], tfull[2], tempty[2], drain;
   __shared__ uint32_t tbase;
   __shared__ int abort_flag;
   volatile int* abort_ = &abort_flag;
@@ -120,6 +120,7 @@ __global__ void __launch_bounds__(HTHREADS, 1)
       mbar_init(&tfull[i], 1);
       mbar_init(&tempty[i], HNEPI);
     }
+    mbar_init(&drain, 1);
     fence_barrier_init();
     prefetch_tmap(&amap);
     prefetch_tmap(&wmap);
@@ -138,6 +139,7 @@ __global__ void __launch_bounds__(HTHREADS, 1)
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
+      ArmedStages armed;
       bool ok = true;
       for (int t = blockIdx.x; t < J.tiles && ok; t += gridDim.x) {
         int lb, nt, mt;
@@ -147,11 +149,14 @@ __global__ void __launch_bounds__(HTHREADS, 1)
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_)) { ok = false; break; }
           unsigned char* a = sm + stage * SB;
           mbar_expect_tx(&full[stage], (uint32_t)SB);
+          armed.arm(stage, phase);
           tma_load_3d(a, &amap, &full[stage], kb * HK, mt * HM, lb);
           tma_load_3d(a + HM * 128, &wmap, &full[stage], kb * HK, nt * J.NT, l);
           if (++stage == HSTAGE) { stage = 0; phase ^= 1u; }
         }
       }
+      // every load issued has landed before the CTA's shared memory goes
+      if (!armed.drain(full)) *abort_ = 1;
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
@@ -159,7 +164,7 @@ __global__ void __launch_bounds__(HTHREADS, 1)
       int stage = 0;
       uint32_t phase = 0, bphase = 0;
       const uint32_t idesc = idesc_bf16_f32(HM, J.NT);
-      bool ok = true;
+      bool ok = true, issued = false;
       for (int t = blockIdx.x, j = 0; t < J.tiles && ok; t += gridDim.x, ++j) {
         const int buf = j & 1;
         if (!mbar_wait(&tempty[buf], ((bphase >> buf) & 1u) ^ 1u, abort_)) break;
@@ -175,9 +180,15 @@ __global__ void __launch_bounds__(HTHREADS, 1)
             mma_bf16(dcol, sdesc_k_sw128(a + w * 32), sdesc_k_sw128(a + HM * 128 + w * 32), idesc,
                      (kb | w) ? 1u : 0u);
           mma_commit(&empty[stage]);
+          issued = true;
           if (++stage == HSTAGE) { stage = 0; phase ^= 1u; }
         }
         if (ok) mma_commit(&tfull[buf]);
+      }
+      // every MMA issued has finished before the CTA's tensor memory goes
+      if (issued) {
+        mma_commit(&drain);
+        if (!mbar_wait_drain(&drain, 0)) *abort_ = 1;
       }
     }
   } else {

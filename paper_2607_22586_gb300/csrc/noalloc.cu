@@ -27,7 +27,8 @@ size_t round256(size_t x) { return (x + 255) & ~size_t(255); }
 
 // Device address of the scratch array on the current device. In host code the
 // symbol only names a host-side stand-in, so the address is looked up once per
-// device with that device current.
+// device with that device current and kept for the life of the process (a
+// later cudaDeviceReset would invalidate it; the header says so).
 cudaError_t scratch_address(void** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);

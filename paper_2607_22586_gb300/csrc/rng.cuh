@@ -30,25 +30,35 @@ __device__ __forceinline__ float uniform_of(uint32_t w) {
   return ((float)(w >> 9) + 0.5f) * 1.1920928955078125e-07f;
 }
 
-// ln(u) for a uniform u = ((w >> 9) + 1/2) 2^-23. Near 1, with c = 1 - u
-// (exact) below 1/16, the series ln(1 - c) = -(c + c^2/2 + ... + c^8/8)
-// (truncation below 1e-11 relative); elsewhere log2(u) from the MUFU times
-// ln 2, whose absolute error (about 2^-22) is small against |ln u| >= 0.064.
+// ln(u) for a uniform u in (0, 1): u = m 2^e with m in [sqrt(1/2), sqrt(2)),
+// ln m = 2 atanh(s) with s = (m - 1) / (m + 1) (|s| <= 0.1716; m - 1 is exact,
+// 1 / (m + 1) from the approximate reciprocal and one Newton step, about one
+// ulp) from the series 2 (s + s^3/3 + ... + s^13/13), whose truncation is
+// below 2e-12 relative, and e ln 2 with ln 2 split into a short leading part
+// (its product with e is exact) and the remainder (the argument reduction of
+// Cody and Waite, 1980). Rounding leaves about 3 float32 ulp of relative
+// error.
 __device__ __forceinline__ float ln_uniform(float u) {
-  const float c = 1.0f - u;
-  float lg;
-  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(lg) : "f"(u));
-  const float far = lg * 0.6931471805599453f;
-  float p = 1.0f / 8.0f;
-  p = fmaf(p, c, 1.0f / 7.0f);
-  p = fmaf(p, c, 1.0f / 6.0f);
-  p = fmaf(p, c, 1.0f / 5.0f);
-  p = fmaf(p, c, 1.0f / 4.0f);
-  p = fmaf(p, c, 1.0f / 3.0f);
-  p = fmaf(p, c, 0.5f);
-  p = fmaf(p, c, 1.0f);
-  const float near = -c * p;
-  return c < 0.0625f ? near : far;
+  const uint32_t bits = __float_as_uint(u);
+  int e = (int)(bits >> 23) - 127;
+  float m = __uint_as_float((bits & 0x7FFFFFu) | 0x3F800000u);   // [1, 2)
+  if (m > 1.41421356f) { m *= 0.5f; ++e; }
+  const float den = m + 1.0f;
+  float rcp;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(rcp) : "f"(den));
+  rcp = fmaf(rcp, fmaf(-den, rcp, 1.0f), rcp);
+  const float s = (m - 1.0f) * rcp;
+  const float t = s * s;
+  float p = 1.0f / 13.0f;
+  p = fmaf(p, t, 1.0f / 11.0f);
+  p = fmaf(p, t, 1.0f / 9.0f);
+  p = fmaf(p, t, 1.0f / 7.0f);
+  p = fmaf(p, t, 1.0f / 5.0f);
+  p = fmaf(p, t, 1.0f / 3.0f);
+  const float s2 = 2.0f * s;
+  const float lnm = fmaf(s2 * t, p, s2);
+  const float fe = (float)e;
+  return fmaf(fe, 0.693145751953125f, fmaf(fe, 1.4286068203094172e-06f, lnm));
 }
 
 // sin(pi x), cos(pi x) for |x| < 1 with x a multiple of 2^-23: x = y + k/2

@@ -30,8 +30,10 @@
 //   accumulator lane is a key, so each thread sums exp2(x - c_row) over the
 //   columns of a group in registers and writes one group mass per key
 //   (coalesced along keys).
-// Every wait is bounded; a CTA that gives up raises the timeout status bit,
-// stops issuing work and still frees its TMEM.
+// Every wait is bounded; a CTA that gives up raises the timeout status bit and
+// stops issuing work. Before it frees its tensor memory and exits, its
+// producer waits (bounded) for every TMA load it armed and its MMA issuer for
+// every MMA it issued, so no copy or MMA lands in memory the CTA gave back.
 #include <cudaTypedefs.h>
 
 #include <algorithm>
@@ -309,9 +311,10 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   unsigned char* sm =
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
   unsigned char* stat = sm;
-  unsigned char* ring = sm + SM::STAT_BYTES;
-  float* cs_all = reinterpret_cast<float*>(ring + SM::RING_BYTES);
+  unsigned char* ring_buf = sm + SM::STAT_BYTES;
+  float* cs_all = reinterpret_cast<float*>(ring_buf + SM::RING_BYTES);
   __shared__ uint64_t full[NSTAGE], empty[NSTAGE], sfull, sempty, tfull[2], tempty[2];
+  __shared__ uint64_t drain, never;
   __shared__ uint32_t tbase;
   __shared__ int abort_flag;
   volatile int* abort_ = &abort_flag;
@@ -337,6 +340,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       mbar_init(&tfull[i], 1);
       mbar_init(&tempty[i], NEPI / 2);   // drained by a pair of warpgroups
     }
+    mbar_init(&drain, 1);
+    mbar_init(&never, 1);                // nothing arrives here (test_stuck_wait)
     fence_barrier_init();
     prefetch_tmap(&kmap);
     prefetch_tmap(&pmap);
@@ -355,6 +360,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0, sphase = 0;
+      ArmedStages armed_k, armed_s;
       long long prev = -1;
       bool ok = true;
       for (int i = 0; i < walk.n && ok; ++i) {
@@ -366,6 +372,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           const Block k = mass_block(P, S, x.tile);
           const int row0 = k.row0, rows = k.rows;
           mbar_expect_tx(&sfull, (uint32_t)(rows * D * 2));
+          armed_s.arm(0, sphase);
           const int zc = (x.l * P.B + x.b) * P.Hkv + x.h;
           for (int c = 0; c < SM::CH; ++c)
             for (int r = 0; r < rows; r += 16)
@@ -377,12 +384,15 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         for (int kt = x.t0; kt < x.t1; kt += BK) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_)) { ok = false; break; }
           mbar_expect_tx(&full[stage], (uint32_t)SM::STAGE_BYTES);
+          armed_k.arm(stage, phase);
           for (int c = 0; c < SM::CH; ++c)
-            tma_load_3d(ring + stage * SM::STAGE_BYTES + c * BK * 128, &kmap, &full[stage],
+            tma_load_3d(ring_buf + stage * SM::STAGE_BYTES + c * BK * 128, &kmap, &full[stage],
                         x.h * D + c * 64, kbase + kt, x.l);
           if (++stage == NSTAGE) { stage = 0; phase ^= 1u; }
         }
       }
+      // every load issued has landed before the CTA's shared memory goes
+      if (!(armed_k.drain(full) && armed_s.drain(&sfull))) *abort_ = 1;
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
@@ -391,7 +401,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       uint32_t phase = 0, bphase = 0, sphase = 0;   // bphase: one phase bit per accumulator
       long long prev = -1;
       uint32_t idesc = 0;
-      bool ok = true;
+      bool ok = true, issued = false;
       for (int i = 0; i < walk.n && ok; ++i) {
         const int u = walk_unit<LISTS>(S, wk, walk, i);
         const Unit x = decode(P, S, u);
@@ -411,7 +421,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           if (!mbar_wait(&full[stage], phase, abort_) ||
               !mbar_wait(&tempty[buf], ((bphase >> buf) & 1u) ^ 1u, abort_)) { ok = false; break; }
           fence_after();
-          const uint32_t ks_base = smem_u32(ring + stage * SM::STAGE_BYTES);
+          const uint32_t ks_base = smem_u32(ring_buf + stage * SM::STAGE_BYTES);
           const uint32_t st_base = smem_u32(stat);
           const uint32_t dcol = tmem + (uint32_t)(buf * ACC_STRIDE);
 #pragma unroll
@@ -423,9 +433,15 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           }
           mma_commit(&empty[stage]);
           mma_commit(&tfull[buf]);
+          issued = true;
           if (++stage == NSTAGE) { stage = 0; phase ^= 1u; }
           bphase ^= 1u << buf;
         }
+      }
+      // every MMA issued has finished before the CTA's tensor memory goes
+      if (issued) {
+        mma_commit(&drain);
+        if (!mbar_wait_drain(&drain, 0)) *abort_ = 1;
       }
     }
   } else {
@@ -443,6 +459,10 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     uint32_t bphase = 0;                  // one phase bit per accumulator
     long long prev_blk = -1;
     bool ok = true;
+    // test only: the first epilogue warp of CTA 0 waits on a barrier that
+    // nothing arrives on, gives up after a few polls and aborts the CTA
+    if (P.test_stuck_wait && blockIdx.x == 0 && ew == 0)
+      ok = mbar_wait(&never, 0, abort_, kTestSpinLimit);
     for (int i = 0; i < walk.n && ok; ++i) {
       const int u = walk_unit<LISTS>(S, wk, walk, i);
       const Unit x = decode(P, S, u);
@@ -535,6 +555,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
   // full / sfull / tempty count on the leader's copies; empty / sempty /
   // tfull receive the leader's multicast commits in both CTAs
   __shared__ uint64_t full[PNSTAGE], empty[PNSTAGE], sfull, sempty, tfull[2], tempty[2];
+  __shared__ uint64_t drain;
   __shared__ uint32_t tbase;
   __shared__ int abort_flag;
   volatile int* abort_ = &abort_flag;
@@ -557,6 +578,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
       mbar_init(&tfull[i], 1);
       mbar_init(&tempty[i], 2 * (NEPI / 32));   // every epilogue warp of both CTAs
     }
+    mbar_init(&drain, 1);
     fence_barrier_init();
     prefetch_tmap(&kmap);
     prefetch_tmap(&pmap);
@@ -576,6 +598,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0, sphase = 0;
+      ArmedStages armed_k, armed_s;   // the leader's barriers count both CTAs' loads
       long long prev = -1;
       bool ok = true;
       for (int i = 0; i < walk.n && ok; ++i) {
@@ -583,7 +606,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
         const long long key = block_key(P, S, x);
         if (key != prev) {
           if (!mbar_wait(&sempty, sphase ^ 1u, abort_)) { ok = false; break; }
-          if (rank == 0) mbar_expect_tx(&sfull, (uint32_t)(2 * PROWS * D * 2));
+          if (rank == 0) {
+            mbar_expect_tx(&sfull, (uint32_t)(2 * PROWS * D * 2));
+            armed_s.arm(0, sphase);
+          }
           const uint32_t bar = mapa(smem_u32(&sfull), 0);
           const int zc = (x.l * P.B + x.b) * P.Hkv + x.h;
           const int row0 = x.tile * SROWS + (int)rank * PROWS;
@@ -596,7 +622,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
         const int kbase = P.req[x.b].tok_off + (int)rank * (PBK / 2);
         for (int kt = x.t0; kt < x.t1; kt += PBK) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_)) { ok = false; break; }
-          if (rank == 0) mbar_expect_tx(&full[stage], (uint32_t)(2 * SM::STAGE_BYTES));
+          if (rank == 0) {
+            mbar_expect_tx(&full[stage], (uint32_t)(2 * SM::STAGE_BYTES));
+            armed_k.arm(stage, phase);
+          }
           const uint32_t bar = mapa(smem_u32(&full[stage]), 0);
           for (int c = 0; c < SM::CH; ++c)
             tma_load_3d_pair(ring + stage * SM::STAGE_BYTES + c * (PBK / 2) * 128, &kmap, bar,
@@ -604,6 +633,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
           if (++stage == PNSTAGE) { stage = 0; phase ^= 1u; }
         }
       }
+      // the leader waits for every load of both CTAs it armed (the pair's
+      // final cluster barrier keeps the peer until then)
+      if (rank == 0 && !(armed_k.drain(full) && armed_s.drain(&sfull))) *abort_ = 1;
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer (leader)
@@ -612,7 +644,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
       uint32_t phase = 0, bphase = 0, sphase = 0;
       long long prev = -1;
       const uint32_t idesc = idesc_bf16_f32(2 * PROWS, PBK);
-      bool ok = true;
+      bool ok = true, issued = false;
       for (int i = 0; i < walk.n && ok; ++i) {
         const Unit x = decode(P, S, walk_unit<LISTS>(S, wk, walk, i));
         const long long key = block_key(P, S, x);
@@ -640,9 +672,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
           }
           mma_commit_pair(&empty[stage], 0x3);
           mma_commit_pair(&tfull[buf], 0x3);
+          issued = true;
           if (++stage == PNSTAGE) { stage = 0; phase ^= 1u; }
           bphase ^= 1u << buf;
         }
+      }
+      // every pair MMA issued has finished before either CTA's tensor memory goes
+      if (issued) {
+        mma_commit_pair(&drain, 0x1);
+        if (!mbar_wait_drain(&drain, 0)) *abort_ = 1;
       }
     }
   } else {

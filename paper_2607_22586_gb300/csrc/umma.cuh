@@ -53,15 +53,47 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Wait until the phase of parity `parity` has completed. Returns false if the
-// wait gave up (spin limit reached, or another role already aborted).
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
-  for (uint32_t i = 0; i < kSpinLimit; ++i) {
+// wait gave up (`limit` polls, or another role already aborted).
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                          uint32_t limit = kSpinLimit) {
+  for (uint32_t i = 0; i < limit; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*abort) return false;
   }
   *abort = 1;
   return false;
 }
+
+// The same wait without the abort check, for the drain at a CTA's exit: the
+// TMA loads and MMAs a role issued must have finished before the CTA's shared
+// and tensor memory are released, whether or not the CTA aborted.
+__device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity) {
+  for (uint32_t i = 0; i < kSpinLimit; ++i)
+    if (mbar_try_wait(bar, parity)) return true;
+  return false;
+}
+
+// Polls of the test-only wait on a barrier that nothing arrives on
+// (mmshift_debug.test_stuck_wait): a few milliseconds at most.
+constexpr uint32_t kTestSpinLimit = 64;
+
+// Loads a producer has armed, per ring stage: bit s of `armed` says stage s
+// was filled at least once, bit s of `parity` is the phase of its last fill.
+// drain() waits for each of those last fills to land (they complete in
+// order, so every earlier one has landed too).
+struct ArmedStages {
+  uint32_t armed = 0, parity = 0;
+  __device__ __forceinline__ void arm(int s, uint32_t phase) {
+    armed |= 1u << s;
+    parity = (parity & ~(1u << s)) | ((phase & 1u) << s);
+  }
+  __device__ __forceinline__ bool drain(uint64_t* bars) const {
+    bool ok = true;
+    for (int s = 0; s < 32; ++s)
+      if ((armed >> s) & 1u) ok = mbar_wait_drain(&bars[s], (parity >> s) & 1u) && ok;
+    return ok;
+  }
+};
 
 // 3-D tiled TMA load into shared memory, completion counted on `bar`.
 __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, uint64_t* bar,

@@ -55,3 +55,33 @@ def test_pyramid_budgets_average_the_uniform_budget():
     assert np.all(np.diff(hb[:, 0, 0]) <= 0)                      # shrinking with depth
     assert abs(hb.mean() - C) <= 1.0                               # C on average
     assert np.all(hb == hb[:, :, :1])                              # equal across heads
+
+
+PEAKS = {"hbm_gbs": 6783.5, "bf16_tflops": 1910.3, "bf16_tflops_sustained": 1704.3,
+         "sm_max_mhz": 2070.0, "clocks_under_load": {"sm_mhz_median": 1447.0}}
+
+
+def test_tensor_peak_follows_the_clock_seen():
+    """A timed region at the maximum SM clock is held to the burst GEMM peak;
+    one whose median clock sat near the sustained run's clock to the
+    sustained peak; with no clock record, the higher (burst) peak."""
+    peak, kind = bench.tensor_peak(PEAKS, {"sm_mhz": 2070.0}, "measured")
+    assert peak == 1910.3 and "burst" in kind
+    peak, kind = bench.tensor_peak(PEAKS, {"sm_mhz": 1500.0}, "measured")
+    assert peak == 1704.3 and "sustained" in kind
+    peak, kind = bench.tensor_peak(PEAKS, None, "measured")
+    assert peak == 1910.3 and "no clock record" in kind
+
+
+def test_score_roofline_recomputes_from_stage_times():
+    """The reported fraction is the pass's algorithmic flops over its event
+    time over the chosen peak: recomputable from stage_ms and the formula."""
+    wl = S.WORKLOADS["qwen7b-28l-32k"]
+    stage = {"softmax_pass": 3.2, "mass_pass": 3.416}
+    roof = bench.score_roofline(wl, PAPER, stage, True, PEAKS, "measured", {"sm_mhz": 2070.0})
+    flops = 2.0 * 128 * (512 * 7 + 7) * 32768 * 4 * 28
+    assert roof["kernel"] == "mass_pass"
+    assert abs(roof["achieved"] - flops / 3.416e-3 / 1e12) < 1e-6
+    assert abs(roof["frac"] - roof["achieved"] / 1910.3) < 1e-12
+    assert abs(roof["frac"] - 0.517) < 0.002
+    assert abs(roof["hbm"]["bytes_per_launch"] - 28 * 33_554_432) < 1

@@ -7,17 +7,20 @@ points (defaults, output rows, workspace size, validation, status strings),
 which need no GPU. It checks that the header is valid C, that the exported
 names link, and that the values match the documented ones.
 """
+import ctypes
 import os
 import shutil
 import subprocess
 
 import pytest
 
+from paper_2607_22586_gb300 import _lib as L
 from paper_2607_22586_gb300 import build as B
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 PROGRAM = r"""
+#include <stddef.h>
 #include <stdio.h>
 #include <string.h>
 #include "mmshift.h"
@@ -53,6 +56,8 @@ int main(void) {
   printf("null_select %d\n", (int)mmshift_select(&s, NULL, NULL, NULL, NULL, &p, NULL, NULL, NULL,
                                                  NULL, NULL, 0, NULL));
   printf("status %s\n", mmshift_status_string(MMSHIFT_ERR_WORKSPACE));
+  printf("sizes %d %d %d %d\n", (int)sizeof(mmshift_params), (int)sizeof(mmshift_shape),
+         (int)sizeof(mmshift_debug), (int)offsetof(mmshift_debug, test_stuck_wait));
   return 0;
 }
 """
@@ -85,3 +90,6 @@ def test_plain_c_program_links_and_runs(tmp_path):
     assert got["bad_window"] == "1"                                # MMSHIFT_ERR_INVALID_ARG
     assert got["null_select"] == "1"
     assert got["status"].strip() != ""
+    # the ctypes binding lays the structs out as the C compiler does
+    assert got["sizes"] == (f"{ctypes.sizeof(L.Params)} {ctypes.sizeof(L.Shape)} "
+                            f"{ctypes.sizeof(L.Debug)} {L.Debug.test_stuck_wait.offset}")

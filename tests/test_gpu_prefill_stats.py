@@ -177,23 +177,24 @@ def test_select_with_prefill_proxies_f32():
                          out_lo=int(outs[b]))
 
 
-def test_select_with_prefill_proxies_bf16_agreement():
-    """bf16: the statistics' fp32 error can move a proxy by one ulp in a few
-    elements; selection must agree with the oracle's on almost every key."""
+def test_select_with_prefill_proxies_bf16():
+    """bf16: the statistics over all prompt queries are float32 sums (their
+    error bound is derived above), which moves the rounding of a few proxy
+    elements (at most 1e-2 of them; an element whose value nearly cancels can
+    move by more than one ulp); the selection must then follow the per-key
+    rule against the oracle re-run on the GPU's proxies."""
     wl = QWEN1
     li = S.make_layer(wl, 0)
     qf = S.make_prompt_queries(wl, 0, li)
     h = PT.hyper(seed=5)
     gpu = _gpu_prefill_select(wl, li, qf, h)
-    ref = _oracle_prefill(wl, li, qf, h)[0]
-    pdiff = np.mean(gpu["proxies"][0, 0] != ref["proxies"])
+    own = _oracle_prefill(wl, li, qf, h)[0]["proxies"]
+    got = gpu["proxies"][0, 0].astype(np.float64)
+    pdiff = np.mean(got != own)
     assert pdiff <= 1e-2, f"{pdiff:.2e} of proxies differ from the oracle's"
-    err = np.abs(gpu["group_mass"][0].astype(np.float64) - ref["group_mass"])
-    bad = err > PT.RTOL * np.abs(ref["group_mass"]) + PT.ATOL
-    assert bad.mean() < 1e-3, f"{bad.mean():.2e} of group masses outside tolerance"
-    for hh in range(wl.n_kv_heads):
-        a, b = set(gpu["idx"][0][:, hh].tolist()), set(ref["idx"][:, hh].tolist())
-        assert len(a & b) >= 0.98 * len(b), f"head {hh}: overlap {len(a & b)}/{len(b)}"
+    refs = PT.oracle_layer(wl, li, h, 0, proxies=gpu["proxies"][0])
+    cu = wl.cu_seqlens()
+    PT.check_request(gpu, refs[0], h, int(cu[0]), int(cu[1]), 0, "prefill bf16 req 0")
 
 
 def test_prefill_stats_full_size_layer_sampled():

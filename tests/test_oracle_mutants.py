@@ -214,6 +214,33 @@ def _topk_heads_drops_last_token(s, head_budgets, capacity):
     return idx, counts
 
 
+_orig_scores = O.scores
+_orig_select_request = O.select_request
+
+
+def _scores_mass_votes(mode, abar, alpha, tau, lam):
+    return _orig_scores(O.SCORE_VOTE, abar, alpha, tau, lam)
+
+
+def _scores_mass_with_anchor(mode, abar, alpha, tau, lam):
+    s = _orig_scores(mode, abar, alpha, tau, lam)
+    return s + lam * alpha if mode == O.SCORE_MASS else s
+
+
+def _select_request_stream_zero(keys, values, qwin, budget, **kw):
+    kw["b"] = 0
+    return _orig_select_request(keys, values, qwin, budget, **kw)
+
+
+def _select_first_budget(keys, values, qwin, cu_seqlens, budgets, proxies=None, **kw):
+    res = []
+    for b in range(len(budgets)):
+        lo, hi = int(cu_seqlens[b]), int(cu_seqlens[b + 1])
+        res.append(O.select_request(keys[lo:hi], values[lo:hi], qwin[b], int(budgets[0]), b=b,
+                                    proxies=None if proxies is None else proxies[b], **kw))
+    return res
+
+
 MUTANTS = {
     "std_ddof0": ("window_stats", _window_stats_ddof0),
     "prefill_std_ddof0": ("prefill_stats", _prefill_stats_ddof0),
@@ -239,6 +266,10 @@ MUTANTS = {
     "coverage_renormalised_on_kept": ("attention_coverage", _coverage_renormalised_on_kept),
     "head_budgets_ignored": ("select_topk_heads", _topk_heads_capacity_everywhere),
     "head_budgets_drop_last_token": ("select_topk_heads", _topk_heads_drops_last_token),
+    "mass_mode_votes": ("scores", _scores_mass_votes),
+    "mass_mode_with_anchor": ("scores", _scores_mass_with_anchor),
+    "request_stream_always_zero": ("select_request", _select_request_stream_zero),
+    "batch_uses_first_budget": ("select", _select_first_budget),
 }
 
 

@@ -436,11 +436,114 @@ def pin_topk_bruteforce(orc=O):
             assert cand == list(bests[0])
 
 
+def pin_mass_scores_bruteforce(orc=O):
+    """MASS scoring (Table 5's "+ Var. Exp." row): S_t is the attention mass
+    of all proxies of the r grouped heads, summed. Against a brute loop over
+    heads, proxies and keys with math.exp (no softmax routine, no grouping);
+    the grouping must not matter, nor the order of the groups, nor the anchor."""
+    keys, proxies, q_last = _tiny_problem(31, t_len=12, hq=4, hkv=2, d=4, n_p=6)
+    t_len, hkv, d = keys.shape
+    hq, n_p, _ = proxies.shape
+    r = hq // hkv
+    scale = 0.7
+    brute = np.zeros((hkv, t_len))
+    for hh in range(hq):
+        for i in range(n_p):
+            lg = [scale * sum(proxies[hh, i, j] * keys[t, hh // r, j] for j in range(d))
+                  for t in range(t_len)]
+            mx = max(lg)
+            ex = [math.exp(x - mx) for x in lg]
+            z = math.fsum(ex)
+            for t in range(t_len):
+                brute[hh // r, t] += ex[t] / z
+    alpha = orc.anchor_attention(q_last, keys, scale)
+    for n_groups in (1, 2, 3, 6):
+        abar = orc.group_masses(proxies, keys, n_groups, scale)
+        for h in range(hkv):
+            s = orc.scores(orc.SCORE_MASS, abar[h], alpha[h], 0.9, 1.0)
+            np.testing.assert_allclose(s, brute[h], rtol=1e-12)
+            rev = orc.scores(orc.SCORE_MASS, abar[h][::-1], alpha[h] * 7.0, 0.5, 3.0)
+            np.testing.assert_allclose(rev, brute[h], rtol=1e-12)
+    # the whole method in MASS mode keeps T-1 and the top C-1 of that mass
+    qwin = np.stack([q_last * 0.3, q_last], axis=0)
+    res = orc.select_request(keys, keys, qwin, 5, n_proxies=n_p, n_groups=3, proxies=proxies,
+                             dtype=orc.F32, softmax_scale=scale, score_mode=orc.SCORE_MASS)
+    np.testing.assert_allclose(res["scores"], brute, rtol=1e-12)
+    for h in range(hkv):
+        top = sorted(range(t_len - 1), key=lambda t: (-brute[h, t], t))[:4]
+        assert res["idx"][:, h].tolist() == sorted(top + [t_len - 1])
+
+
+def pin_request_streams_and_slicing(orc=O):
+    """A packed batch (Algorithm 1 runs per request): request b draws its
+    proxies from Philox counter (i*d/8 + q, hq, b, layer) -- pinned against
+    numpy's independent Philox and a Box-Muller written out with math.log /
+    math.cos -- and each request's result depends only on its own slice of
+    keys, queries and budget."""
+    seed, layer, hq_n, n_p, d = 5, 3, 2, 3, 16
+    nq = d // 8
+    for b in (0, 1, 4):
+        z = orc.proxy_normals(seed, layer, b, hq_n, n_p, d)
+        for hq in range(hq_n):
+            for i in range(n_p):
+                for q in range(nq):
+                    c0 = i * nq + q
+                    if c0 == 0:
+                        continue   # numpy would carry c0 - 1 into the next word
+                    # numpy's Philox advances the counter before its first block
+                    bg = np.random.Philox(key=[seed, 0], counter=[c0 - 1, hq, b, layer])
+                    raw = bg.random_raw(4)
+                    words = []
+                    for v in raw.tolist():
+                        words += [v & 0xFFFFFFFF, v >> 32]
+                    u = [((w >> 9) + 0.5) * 2.0 ** -23 for w in words]
+                    want = []
+                    for m in range(4):
+                        rad = math.sqrt(-2.0 * math.log(u[2 * m]))
+                        ang = 2.0 * math.pi * u[2 * m + 1]
+                        want += [rad * math.cos(ang), rad * math.sin(ang)]
+                    got = [z[hq, i, 4 * q + k] for k in range(4)] + \
+                          [z[hq, i, d // 2 + 4 * q + k] for k in range(4)]
+                    np.testing.assert_allclose(got, want, rtol=1e-12, atol=1e-13)
+    # slicing: three requests packed; request results depend on their own slice
+    rng = np.random.default_rng(33)
+    hq, hkv, d, w = 4, 2, 8, 3
+    lens, budgets = (9, 14, 6), (4, 20, 2)
+    cu = np.concatenate([[0], np.cumsum(lens)])
+    keys = rng.normal(size=(cu[-1], hkv, d))
+    vals = rng.normal(size=(cu[-1], hkv, d))
+    qwin = rng.normal(size=(3, w, hq, d))
+    kw = dict(n_proxies=8, n_groups=2, seed=2, layer_id=1, dtype=orc.F32, tau=0.9)
+    res = orc.select(keys, vals, qwin, cu, budgets, **kw)
+    keys2 = keys.copy()
+    keys2[cu[0]:cu[1]] = rng.normal(size=(lens[0], hkv, d))   # change request 0 only
+    qwin2 = qwin.copy()
+    qwin2[0] = rng.normal(size=(w, hq, d))
+    res2 = orc.select(keys2, vals, qwin2, cu, budgets, **kw)
+    for b in (1, 2):
+        for k in ("proxies", "group_mass", "scores", "idx", "out_k", "out_v"):
+            np.testing.assert_array_equal(res2[b][k], res[b][k])
+    assert not np.array_equal(res2[0]["group_mass"], res[0]["group_mass"])
+    for b in range(3):
+        assert res[b]["idx"].shape == (min(budgets[b], lens[b]), hkv)
+        assert res[b]["idx"].max() == lens[b] - 1 and res[b]["idx"].min() >= 0
+        # kept rows are the request's own rows
+        lo = cu[b]
+        h = np.arange(hkv)[None]
+        np.testing.assert_array_equal(res[b]["out_v"], vals[lo + res[b]["idx"], h])
+    # the same request content at another batch position draws other proxies
+    alone = orc.select_request(keys[cu[1]:cu[2]], vals[cu[1]:cu[2]], qwin[1], budgets[1], b=0, **kw)
+    assert not np.array_equal(alone["proxies"], res[1]["proxies"])
+    alone1 = orc.select_request(keys[cu[1]:cu[2]], vals[cu[1]:cu[2]], qwin[1], budgets[1], b=1, **kw)
+    np.testing.assert_array_equal(alone1["proxies"], res[1]["proxies"])
+
+
 ALL_PINS = [pin_philox_vs_numpy, pin_normals_distribution, pin_window_stats, pin_prefill_stats,
             pin_hidden_proxies, pin_attention_coverage, pin_head_budgets,
             pin_sampler_closed_form, pin_rope, pin_round_bf16, pin_mass_totals,
             pin_sigma_zero_single_query, pin_shift_and_permutation, pin_budget_ge_t,
-            pin_lastattn, pin_uniform_keys, pin_cover_bruteforce, pin_topk_bruteforce]
+            pin_lastattn, pin_uniform_keys, pin_cover_bruteforce, pin_topk_bruteforce,
+            pin_mass_scores_bruteforce, pin_request_streams_and_slicing]
 
 
 @pytest.mark.parametrize("pin", ALL_PINS, ids=[p.__name__ for p in ALL_PINS])

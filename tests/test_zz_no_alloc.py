@@ -61,6 +61,31 @@ def test_noalloc_matches_workspace_entry_point_on_two_calls():
         assert torch.equal(sc_b, sc_ref)
 
 
+@pytest.mark.gpu
+def test_noalloc_mass_mode_scores_in_scratch():
+    """MASS scoring (no vote, no anchor): the scores live in the static array
+    where the vote's bitmaps would start; twice in a row, equal to the
+    workspace entry point."""
+    wl, h, gm, _ = _case(13, (2500, 900, 3), (300, 128, 1), 8, 0.95)
+    h = dict(h, score_mode=L.MMSHIFT_SCORE_MASS)
+    shape = PT.shape_of(wl)
+    params = PT.abi_params(h)
+    rows = M.mmshift_output_rows(shape)
+    hkv, T = wl.n_kv_heads, wl.total_tokens
+    gm_d = torch.from_numpy(gm).cuda()
+    ws_bytes = M.mmshift_workspace_size(shape, params)
+    ws = torch.zeros(ws_bytes, dtype=torch.uint8, device="cuda")
+    idx_ref = torch.full((1, rows, hkv), -1, dtype=torch.int32, device="cuda")
+    sc_ref = torch.empty((1, hkv, T), device="cuda")
+    M.check(M.mmshift_scores_topk(shape, params, gm_d, None, sc_ref, idx_ref, ws, ws_bytes),
+            "scores_topk mass")
+    for _ in range(2):
+        idx = torch.full((1, rows, hkv), -1, dtype=torch.int32, device="cuda")
+        M.check(M.mmshift_scores_topk_noalloc(shape, params, gm_d, None, None, idx), "noalloc mass")
+        torch.cuda.synchronize()
+        assert torch.equal(idx, idx_ref)
+
+
 def test_noalloc_rejects_problem_larger_than_its_scratch():
     # 8 KV heads x 32 groups x 300K tokens of bitmaps + scores exceed 8 MiB;
     # refused by host-side validation before any device work
