@@ -129,8 +129,12 @@ mmshift_status build_problem(const mmshift_shape* s, const mmshift_params* p, Pr
 }
 
 struct Layout {
-  size_t status, packed, part, cvals, gmass, anchor, bits, scores, refine, refine_stats, total;
+  size_t status, packed, part, cvals, gmass, anchor, alog, bits, scores, refine, refine_stats, total;
 };
+
+// The anchor rows start a 256-row block of their own: on the tensor-core
+// path the softmax pass leaves them out (Problem::anchor_split).
+bool anchor_spills(const Problem& P) { return P.G > 0 && P.n_group_rows % kRowTile == 0; }
 
 Layout layout_of(const Problem& P) {
   const size_t esz = P.dtype == MMSHIFT_BF16 ? 2 : 4;
@@ -143,6 +147,7 @@ Layout layout_of(const Problem& P) {
   w.cvals = o;  o += align256(L * P.B * P.Hkv * (size_t)P.Prows_pad * sizeof(float));
   w.gmass = o;  o += align256(L * P.Hkv * (size_t)P.G * P.total_T * sizeof(float));
   w.anchor = o; o += align256(L * P.Hkv * (size_t)P.total_T * sizeof(float));
+  w.alog = o;   o += anchor_spills(P) ? align256(L * P.Hkv * (size_t)P.r * P.total_T * sizeof(float)) : 0;
   w.bits = o;   o += align256(L * P.Hkv * (size_t)P.G * P.total_words * sizeof(uint32_t));
   w.scores = o; o += align256(L * P.Hkv * (size_t)P.total_T * sizeof(float));
   // count word, the list of proxy elements to recompute in float64, then the
@@ -165,6 +170,7 @@ mmshift_status carve(const Problem& P, void* ws, size_t bytes, Buffers* bf) {
   bf->cvals = reinterpret_cast<float*>(base + w.cvals);
   bf->gmass = reinterpret_cast<float*>(base + w.gmass);
   bf->anchor = reinterpret_cast<float*>(base + w.anchor);
+  bf->alog = reinterpret_cast<float*>(base + w.alog);
   bf->bits = reinterpret_cast<uint32_t*>(base + w.bits);
   bf->scores = reinterpret_cast<float*>(base + w.scores);
   bf->refine_count = reinterpret_cast<int*>(base + w.refine);
@@ -204,6 +210,14 @@ StageMarks marks_of(const mmshift_debug* dbg, cudaStream_t st) {
 // needs a 16-byte aligned base) allow it; CUDA-core scoring otherwise.
 int choose_umma(const Problem& P, const void* K) {
   return (umma_supported(P) && (reinterpret_cast<uintptr_t>(K) & 15) == 0) ? 1 : 0;
+}
+
+// Scoring path of a call: tensor or CUDA cores, and the softmax partials
+// and anchor handling that go with it.
+void set_score_path(Problem& P, const void* K) {
+  P.use_umma = choose_umma(P, K);
+  P.part_slots = P.use_umma ? kUmmaPartSlots : 1;
+  P.anchor_split = P.use_umma && anchor_spills(P) ? 1 : 0;
 }
 
 // Kernels one mmshift_select call enqueues (reported through mmshift_debug).
@@ -332,8 +346,7 @@ static mmshift_status select_impl(const mmshift_shape* s, const void* K, const v
   mmshift_status st = prepare(s, p, &P);
   if (st != MMSHIFT_OK) return st;
   if (!p || !K || !V || !Qwin || !out_idx || !out_K || !out_V) return MMSHIFT_ERR_INVALID_ARG;
-  P.use_umma = choose_umma(P, K);
-  P.part_slots = P.use_umma ? kUmmaPartSlots : 1;
+  set_score_path(P, K);
   Buffers bf;
   if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
   // K and Qwin are streamed by every pass: device memory; V is read only for
@@ -539,8 +552,7 @@ mmshift_status mmshift_proxy_mass(const mmshift_shape* s, const void* K, const v
   mmshift_status st = prepare(s, p, &P);
   if (st != MMSHIFT_OK) return st;
   if (!p || !K || !Qwin || !anchor || (P.G && !group_mass)) return MMSHIFT_ERR_INVALID_ARG;
-  P.use_umma = choose_umma(P, K);
-  P.part_slots = P.use_umma ? kUmmaPartSlots : 1;
+  set_score_path(P, K);
   Buffers bf;
   if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
   bf.proxies_in = proxies;
@@ -678,8 +690,7 @@ mmshift_status mmshift_coverage(const mmshift_shape* s, const void* K, const voi
   Problem P;
   if ((st = prepare(s, &p, &P)) != MMSHIFT_OK) return st;
   if (!K || !Qwin || !dec_q || !idx || !cov) return MMSHIFT_ERR_INVALID_ARG;
-  P.use_umma = choose_umma(P, K);
-  P.part_slots = P.use_umma ? kUmmaPartSlots : 1;
+  set_score_path(P, K);
   Buffers bf;
   if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
   bf.proxies_in = dec_q;

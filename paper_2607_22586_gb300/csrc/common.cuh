@@ -52,6 +52,11 @@ struct Problem {
   float rope_theta;
   int32_t rope_off;
   int32_t use_umma;    // steps 2-4 on the tensor cores (set per call)
+  // tensor-core path whose anchor rows would fill a 256-row softmax block of
+  // their own (the group rows end on a block boundary): the softmax pass
+  // leaves them out, the mass pass writes their scaled logits to alog and
+  // anchor_norm_kernel normalises them (set per call)
+  int32_t anchor_split;
   int32_t test_stuck_wait; // test only: see mmshift_debug.test_stuck_wait
   ReqInfo req[MMSHIFT_MAX_BATCH];
 };
@@ -65,6 +70,7 @@ struct Buffers {
   float* cvals;       // [L][B][Hkv][Prows_pad] log2 normaliser of each row
   float* gmass;       // [L][Hkv][G][T]
   float* anchor;      // [L][Hkv][T]
+  float* alog;        // [L][Hkv][r][T] scaled anchor logits (anchor_split only)
   uint32_t* bits;     // [L][Hkv][G][total_words] coverage bitmaps
   float* scores;      // [L][Hkv][T]
   float* mass;        // [L][Hkv][T] or null

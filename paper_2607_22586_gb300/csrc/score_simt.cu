@@ -116,7 +116,8 @@ __global__ void merge_kernel(Problem P, Buffers bf) {
   const int p = blockIdx.x * blockDim.x + threadIdx.x;
   const int bh = blockIdx.y, l = blockIdx.z;
   const int b = bh / P.Hkv, h = bh - b * P.Hkv;
-  if (p >= P.Prows_pad) return;
+  // with anchor_split the softmax pass has no partials for the anchor rows
+  if (p >= (P.anchor_split ? P.n_group_rows : P.Prows_pad)) return;
   const ReqInfo R = P.req[b];
   float m = -INFINITY, z = 0.f;
   const float2* src =

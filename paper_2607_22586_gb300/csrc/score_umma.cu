@@ -498,9 +498,23 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         const bool my_anchor = blk.anchor && (blk.ng == 0 ? sub == 0 : sub == 1);
         if (my_anchor) {
           const int a0 = blk.ng * P.RG;
-          const float sm = group_sum(tacc + (uint32_t)a0, cv + a0, P.anchor_rows, alpha);
-          if (valid)
-            bf.anchor[((size_t)x.l * P.Hkv + x.h) * P.total_T + col] = sm / (float)P.r;
+          if (P.anchor_split) {
+            // no normalisers yet: the scaled logits go to alog, row by row
+            // (coalesced along keys), for anchor_norm_kernel
+            float v[16];
+            tmem_ld16(tacc + (uint32_t)a0, v);
+            tmem_wait_ld();
+            if (valid) {
+              float* dst = bf.alog + ((size_t)x.l * P.Hkv + x.h) * P.r * P.total_T + col;
+#pragma unroll
+              for (int j = 0; j < 16; ++j)
+                if (j < P.r) dst[(size_t)j * P.total_T] = v[j] * alpha;
+            }
+          } else {
+            const float sm = group_sum(tacc + (uint32_t)a0, cv + a0, P.anchor_rows, alpha);
+            if (valid)
+              bf.anchor[((size_t)x.l * P.Hkv + x.h) * P.total_T + col] = sm / (float)P.r;
+          }
         }
         fence_before();
         mbar_arrive(&tempty[buf]);
@@ -756,12 +770,57 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
   if (threadIdx.x == 0 && abort_flag) set_status(bf.status, kStatusTimeout);
 }
 
+// ---------------------------------------------------------------- anchor rows (anchor_split)
+// The anchor is the last window query's attention over the request's keys,
+// averaged over the r query heads of the KV head (Section 3.2.3). With
+// anchor_split its logits come from the mass pass (alog, already scaled to
+// log2 units); here, per (KV head, request, layer): c_j = log2 sum_t
+// exp2(y_jt) for each anchor row j, then anchor_t = (sum_j exp2(y_jt - c_j))
+// / r. The reductions run in a fixed order (thread strides, then xor
+// shuffles, then warps in order), so the result does not depend on the other
+// units of the call.
+constexpr int ANT = 256;
+
+__global__ void __launch_bounds__(ANT) anchor_norm_kernel(const __grid_constant__ Problem P,
+                                                          Buffers bf) {
+  const int h = blockIdx.x, b = blockIdx.y, l = blockIdx.z;
+  const ReqInfo R = P.req[b];
+  const int n = R.t_len, tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  const float* y0 = bf.alog + ((size_t)l * P.Hkv + h) * P.r * P.total_T + R.tok_off;
+  __shared__ float wm[ANT / 32][16], wz[ANT / 32][16], cs[16];
+  for (int j = 0; j < P.r; ++j) {
+    const float* y = y0 + (size_t)j * P.total_T;
+    float m = -INFINITY, z = 0.f;
+    for (int t = tid; t < n; t += ANT) merge_ms(m, z, y[t], 1.f);
+    for (int off = 16; off; off >>= 1) {
+      const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+      const float z2 = __shfl_xor_sync(0xffffffffu, z, off);
+      merge_ms(m, z, m2, z2);
+    }
+    if (lane == 0) { wm[w][j] = m; wz[w][j] = z; }
+  }
+  __syncthreads();
+  if (tid < P.r) {
+    float m = -INFINITY, z = 0.f;
+    for (int i = 0; i < ANT / 32; ++i) merge_ms(m, z, wm[i][tid], wz[i][tid]);
+    cs[tid] = m + __log2f(z);
+  }
+  __syncthreads();
+  float* out = bf.anchor + ((size_t)l * P.Hkv + h) * P.total_T + R.tok_off;
+  for (int t = tid; t < n; t += ANT) {
+    float sm = 0.f;
+    for (int j = 0; j < P.r; ++j) sm += fast_exp2(y0[(size_t)j * P.total_T + t] - cs[j]);
+    out[t] = sm / (float)P.r;
+  }
+}
+
 // ---------------------------------------------------------------- host side
 Sched make_sched(const Problem& P, int pass) {
   Sched s;
   memset(&s, 0, sizeof(s));
   if (pass == 1) {
-    s.ntiles = P.Prows_pad / SROWS;
+    // with anchor_split the anchor rows stay out (they would fill a block alone)
+    s.ntiles = (P.anchor_split ? P.n_group_rows : P.Prows_pad) / SROWS;
   } else {
     // fewest blocks of whole groups, the last one with the anchor rows
     const int per_block = SROWS / P.RG;                      // >= 1 (RG <= SROWS)
@@ -842,6 +901,10 @@ cudaError_t launch_d(const Problem& P, const Buffers& bf, cudaStream_t st, const
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
+  if (P.anchor_split && P.total_T) {
+    anchor_norm_kernel<<<dim3(P.Hkv, P.B, P.L), ANT, 0, st>>>(P, bf);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
   return cudaSuccess;
 }
 
@@ -887,7 +950,7 @@ bool umma_supported(const Problem& P) {
   return major == 10 && tmap_encoder_available();
 }
 
-int umma_launches(const Problem& P) { (void)P; return 3; }
+int umma_launches(const Problem& P) { return P.anchor_split ? 4 : 3; }
 
 cudaError_t launch_score_umma(const Problem& P, const Buffers& bf, cudaStream_t st,
                               const void* K, cudaEvent_t* ev) {

@@ -25,14 +25,14 @@
 namespace mmshift {
 namespace {
 
-constexpr int NT = 512;           // threads per top-k CTA
-constexpr int NW = NT / 32;
-constexpr int NTC = 256;          // threads per coverage CTA
+constexpr int kTopkCand = 4096;   // first-digit candidates a top-k CTA keeps in shared memory
+constexpr int kCoverCand = 6144;  // first-digit candidates a coverage CTA keeps in shared memory
 constexpr int NBIN = 256;
 constexpr int kMaxStaged = 40960; // top-k keys staged in shared memory (160 KB)
 
-template <int NTH>
-constexpr int hist_words() { return 3 * (NTH / 32) * NBIN; }  // per-warp count / weight lo / hi
+// per-warp histograms: counts, and for the weighted select weight lo / hi
+template <int NTH, bool WEIGHTED>
+__host__ __device__ constexpr int hist_words() { return (WEIGHTED ? 3 : 1) * (NTH / 32) * NBIN; }
 
 __device__ __forceinline__ uint32_t ordered_key(float x) {
   uint32_t u = __float_as_uint(x + 0.0f);  // -0 -> +0
@@ -59,6 +59,7 @@ struct SelShared {
   unsigned int prefix;
   unsigned int n_theta;
   unsigned int max_key;
+  unsigned int ncand;
   int aux;
 };
 
@@ -256,28 +257,31 @@ __device__ __forceinline__ void digit_scan(unsigned long long target_w, unsigned
   }
 }
 
-// Smallest prefix of the (key desc, index asc) order whose cumulative weight
-// is >= target_w and whose length is >= target_n (all keys are of
-// non-negative values). On return S.prefix is the key theta of the prefix's
-// last element, S.cum_w / S.cum_n the weight / count of keys above theta and
-// S.n_theta the number of keys equal to theta. Weighted mode: target_w is
-// min(total, ceil(tau * total)) of the exact fixed-point total (S.total), and
-// *shift is lowered (and the first pass redone) if 2^shift units could
-// overflow 64 bits. `hist` is hist_words<NTH>() words of shared memory.
+// Digit passes [p0, p1) of a radix select for the smallest prefix of the
+// (key desc, index asc) order whose cumulative weight is >= target_w and
+// whose length is >= target_n (all keys are of non-negative values). Pass 0
+// starts from prefix 0x80000000; each pass appends its chosen digit to
+// `prefix`. After the last pass, prefix is the key theta of the prefix's last
+// element, S.cum_w / S.cum_n the weight / count of keys above theta and
+// S.n_theta the number of keys equal to theta; after pass 0, S.n_theta is
+// the number of keys that share the chosen first digit (the only keys the
+// later passes look at). Weighted mode: pass 0 sets target_w to
+// min(total, ceil(tau * total)) of the exact fixed-point total (S.total) and
+// lowers *shift (redoing the pass) if 2^shift units could overflow 64 bits.
+// `hist` is hist_words<NTH, WEIGHTED>() words of shared memory.
 template <bool WEIGHTED, int NTH>
-__device__ void radix_select(const KeySrc& get, int n, unsigned long long target_w,
-                             unsigned target_n, int* shift, float tau, SelShared<NTH>& S,
-                             uint32_t* hist) {
+__device__ void radix_passes(const KeySrc& get, int n, int p0, int p1, uint32_t& prefix,
+                             unsigned long long& target_w, unsigned target_n, int* shift,
+                             float tau, SelShared<NTH>& S, uint32_t* hist) {
   constexpr int NWH = NTH / 32;
   const int tid = threadIdx.x;
-  if (tid == 0) { S.cum_w = 0; S.cum_n = 0; }
-  uint32_t prefix = 0x80000000u;
-  constexpr int kSh[4] = {23, 15, 7, 0};
-  constexpr int kWid[4] = {8, 8, 8, 7};
+  if (p0 == 0 && tid == 0) { S.cum_w = 0; S.cum_n = 0; }
 #pragma unroll 1
-  for (int pass = 0; pass < 4; ++pass) {
-    const int sh = kSh[pass], hs = sh + kWid[pass];
-    const uint32_t dmask = (1u << kWid[pass]) - 1u;
+  for (int pass = p0; pass < p1; ++pass) {
+    // digits: bits 23-30 (the exponent), 15-22, 7-14, 0-6
+    const int wid = pass == 3 ? 7 : 8;
+    const int sh = pass == 3 ? 0 : 23 - 8 * pass, hs = sh + wid;
+    const uint32_t dmask = (1u << wid) - 1u;
     digit_histogram<WEIGHTED, NTH>(get, n, prefix, sh, hs, dmask, WEIGHTED ? *shift : 0,
                                    pass == 0, S, hist);
     if (WEIGHTED && pass == 0) {
@@ -303,25 +307,107 @@ __device__ void radix_select(const KeySrc& get, int n, unsigned long long target
     prefix |= (S.digit & dmask) << sh;
     __syncthreads();
   }
-  if (tid == 0) S.prefix = prefix;
+}
+
+template <bool WEIGHTED, int NTH>
+__device__ void radix_select(const KeySrc& get, int n, unsigned long long target_w,
+                             unsigned target_n, int* shift, float tau, SelShared<NTH>& S,
+                             uint32_t* hist) {
+  uint32_t prefix = 0x80000000u;
+  radix_passes<WEIGHTED, NTH>(get, n, 0, 4, prefix, target_w, target_n, shift, tau, S, hist);
+  if (threadIdx.x == 0) S.prefix = prefix;
   __syncthreads();
 }
 
-__global__ void __launch_bounds__(NTC, 4) cover_kernel(Problem P, Buffers bf) {
+// Copies the keys of get[0, n) whose bits at and above `hs` equal those of
+// `prefix` into cand (in no particular order) and returns their number to
+// every thread. Used after the first digit pass, when the keys sharing the
+// chosen first digit fit in shared memory: the later passes then read only
+// them. Each warp appends a ballot's worth at a time.
+template <int NTH>
+__device__ int compact_prefix(const KeySrc& get, int n, uint32_t prefix, int hs, uint32_t* cand,
+                              SelShared<NTH>& S) {
+  const int tid = threadIdx.x, lane = tid & 31;
+  if (tid == 0) S.ncand = 0;
+  __syncthreads();
+  const uint32_t want = prefix >> hs;
+  const unsigned below = (1u << lane) - 1u;
+  auto put = [&](uint32_t k, bool valid) {
+    const bool m = valid && (k >> hs) == want;
+    const unsigned bal = __ballot_sync(0xffffffffu, m);
+    if (!bal) return;
+    unsigned base = 0;
+    if (lane == 0) base = atomicAdd(&S.ncand, (unsigned)__popc(bal));
+    base = __shfl_sync(0xffffffffu, base, 0);
+    if (m) cand[base + __popc(bal & below)] = k;
+  };
+  int done = 0;
+  if (!get.smem && (reinterpret_cast<uintptr_t>(get.gmem) & 15) == 0) {
+    constexpr int U4 = 4;
+    const float4* g4 = reinterpret_cast<const float4*>(get.gmem);
+    const int n4 = n >> 2;
+    for (int base = 0; base < n4; base += U4 * NTH) {
+      float4 f[U4];
+#pragma unroll
+      for (int j = 0; j < U4; ++j) {
+        const int i4 = base + j * NTH + tid;
+        f[j] = i4 < n4 ? __ldg(g4 + i4) : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int j = 0; j < U4; ++j) {
+        const bool valid = base + j * NTH + tid < n4;
+        put(nonneg_key(f[j].x), valid);
+        put(nonneg_key(f[j].y), valid);
+        put(nonneg_key(f[j].z), valid);
+        put(nonneg_key(f[j].w), valid);
+      }
+    }
+    done = n4 << 2;
+  }
+  constexpr int U = 8;
+  for (int base = done; base < n; base += U * NTH) {
+    uint32_t kk[U];
+#pragma unroll
+    for (int j = 0; j < U; ++j) {
+      const int i = base + j * NTH + tid;
+      kk[j] = i < n ? get(i) : 0u;
+    }
+#pragma unroll
+    for (int j = 0; j < U; ++j) put(kk[j], base + j * NTH + tid < n);
+  }
+  __syncthreads();
+  return (int)S.ncand;
+}
+
+template <int NTH>
+__global__ void __launch_bounds__(NTH, 1024 / NTH) cover_kernel(Problem P, Buffers bf) {
   extern __shared__ uint32_t dyn[];
   uint32_t* hist = dyn;
-  __shared__ SelShared<NTC> S;
-  constexpr int NWC = NTC / 32;
+  uint32_t* cand = dyn + hist_words<NTH, true>();   // kCoverCand keys
+  __shared__ SelShared<NTH> S;
+  constexpr int NWC = NTH / 32;
   const int g = blockIdx.x % P.G, h = blockIdx.x / P.G, b = blockIdx.y, l = blockIdx.z;
   const ReqInfo R = P.req[b];
   const int n = R.t_len, tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
   const size_t row = ((size_t)l * P.Hkv + h) * P.G + g;
   const float* m = bf.gmass + row * P.total_T + R.tok_off;
-  // masses are read from L2 in every pass (the working set of the resident
-  // CTAs fits), which keeps shared memory small and four CTAs per SM
+  // the first digit pass reads the masses from L2 / DRAM; when the keys that
+  // share the chosen first digit fit in shared memory they are copied there
+  // and the last three passes read only them
   KeySrc get{nullptr, m};
   int shift = 40;
-  radix_select<true, NTC>(get, n, 0ull, 1u, &shift, P.tau, S, hist);
+  uint32_t prefix = 0x80000000u;
+  unsigned long long target_w = 0;
+  radix_passes<true, NTH>(get, n, 0, 1, prefix, target_w, 1u, &shift, P.tau, S, hist);
+  if (S.n_theta <= (unsigned)kCoverCand) {
+    const int nc = compact_prefix<NTH>(get, n, prefix, 23, cand, S);
+    radix_passes<true, NTH>(KeySrc{cand, nullptr}, nc, 1, 4, prefix, target_w, 1u, &shift, P.tau,
+                            S, hist);
+  } else {
+    radix_passes<true, NTH>(get, n, 1, 4, prefix, target_w, 1u, &shift, P.tau, S, hist);
+  }
+  if (tid == 0) S.prefix = prefix;
+  __syncthreads();
   const uint32_t theta = S.prefix;
   const unsigned n_theta = S.n_theta;
   const unsigned long long target =
@@ -342,7 +428,7 @@ __global__ void __launch_bounds__(NTC, 4) cover_kernel(Problem P, Buffers bf) {
       const int i = base + lane;
       cnt += __popc(__ballot_sync(0xffffffffu, i < hi && get(i) == theta));
     }
-    const unsigned before = warp_excl_prefix<NTC>(S, cnt);
+    const unsigned before = warp_excl_prefix<NTH>(S, cnt);
     if (before < n_tie && before + cnt >= n_tie) {
       unsigned seen = before;
       for (int base = lo; base < hi; base += 32) {
@@ -363,42 +449,46 @@ __global__ void __launch_bounds__(NTC, 4) cover_kernel(Problem P, Buffers bf) {
   const int tstar = S.aux;
   uint32_t* bits = bf.bits + row * P.total_words + R.word_off;
   constexpr int U = 8;
-  for (int base = w * 32; base < n; base += U * NTC) {
+  for (int base = w * 32; base < n; base += U * NTH) {
     uint32_t kk[U];
 #pragma unroll
     for (int j = 0; j < U; ++j) {
-      const int i = base + j * NTC + lane;
+      const int i = base + j * NTH + lane;
       kk[j] = i < n ? get(i) : 0u;
     }
 #pragma unroll
     for (int j = 0; j < U; ++j) {
-      const int i = base + j * NTC + lane;
+      const int i = base + j * NTH + lane;
       const bool mem = i < n && (kk[j] > theta || (kk[j] == theta && i <= tstar));
       const unsigned word = __ballot_sync(0xffffffffu, mem);
-      if (lane == 0 && base + j * NTC < n) bits[(base + j * NTC) >> 5] = word;
+      if (lane == 0 && base + j * NTH < n) bits[(base + j * NTH) >> 5] = word;
     }
   }
 }
 
 // from_scores: S comes from bf.scores as given; otherwise it is built here.
+// NT threads per CTA (512, or 1024 when the units are fewer than the SMs).
+template <int NT>
 __global__ void __launch_bounds__(NT, 1) topk_kernel(Problem P, Buffers bf, int32_t* out_idx,
-                                                     int from_scores) {
+                                                     int from_scores, int staged_cap) {
+  constexpr int NW = NT / 32;
   extern __shared__ uint32_t dyn[];
   uint32_t* hist = dyn;
-  uint32_t* keys_sm = dyn + hist_words<NT>();
+  uint32_t* cand = dyn + hist_words<NT, false>();     // kTopkCand first-digit candidates
+  uint32_t* keys_sm = cand + kTopkCand;               // staged_cap keys
   __shared__ SelShared<NT> S;
   const int h = blockIdx.x, b = blockIdx.y, l = blockIdx.z;
   const ReqInfo R = P.req[b];
   const int n = R.t_len, tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
   const size_t hrow = ((size_t)l * P.Hkv + h) * P.total_T + R.tok_off;
   float* sc = bf.scores + hrow;
-  const bool staged = n <= kMaxStaged;
+  const bool staged = n <= staged_cap;
   if (!from_scores) {
     const float* an = bf.anchor + hrow;
     const uint32_t* bw = bf.bits + ((size_t)l * P.Hkv + h) * P.G * P.total_words + R.word_off;
     // each warp takes 32 consecutive keys at a time, UB chunks of them with
     // their loads in flight together
-    constexpr int UB = 8;
+    constexpr int UB = NT >= 1024 ? 4 : 8;
     for (int base0 = w * 32; base0 < n; base0 += UB * NT) {
       float sv[UB];
       if (P.mode == MMSHIFT_SCORE_VOTE) {
@@ -475,8 +565,18 @@ __global__ void __launch_bounds__(NT, 1) topk_kernel(Problem P, Buffers bf, int3
   }
   KeySrc get{staged ? keys_sm : nullptr, sc};
   const int nc = n - 1;  // candidates t < T-1
-  radix_select<false, NT>(get, nc, 0ull, (unsigned)(keep - 1), nullptr, 0.f, S, hist);
-  const uint32_t theta = S.prefix;
+  // first digit over all candidates; the later digits over the keys that
+  // share it, copied to shared memory when they fit
+  uint32_t theta = 0x80000000u;
+  unsigned long long no_w = 0;
+  radix_passes<false, NT>(get, nc, 0, 1, theta, no_w, (unsigned)(keep - 1), nullptr, 0.f, S, hist);
+  if (S.n_theta <= (unsigned)kTopkCand) {
+    const int ncand = compact_prefix<NT>(get, nc, theta, 23, cand, S);
+    radix_passes<false, NT>(KeySrc{cand, nullptr}, ncand, 1, 4, theta, no_w, (unsigned)(keep - 1),
+                            nullptr, 0.f, S, hist);
+  } else {
+    radix_passes<false, NT>(get, nc, 1, 4, theta, no_w, (unsigned)(keep - 1), nullptr, 0.f, S, hist);
+  }
   const unsigned n_tie = (unsigned)(keep - 1) - S.cum_n;
   // ordered compaction over warp segments
   const int seg = ((nc + NW * 32 - 1) / (NW * 32)) * 32;
@@ -558,23 +658,52 @@ cudaError_t launch_mass_sum(const Problem& P, const Buffers& bf, cudaStream_t st
 
 cudaError_t launch_cover(const Problem& P, const Buffers& bf, cudaStream_t st) {
   if (P.G == 0) return cudaSuccess;
-  const size_t smem = (size_t)hist_words<NTC>() * sizeof(uint32_t);
   dim3 grid(P.Hkv * P.G, P.B, P.L);
-  cover_kernel<<<grid, NTC, smem, st>>>(P, bf);
-  return cudaGetLastError();
+  // few units (the few-proxy setting): 512 threads each, all resident at
+  // two per SM; many units: 256 threads each, four per SM
+  int dev = 0, nsm = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  const long long units = (long long)grid.x * grid.y * grid.z;
+#define MMSHIFT_COVER(NTH)                                                                    \
+  {                                                                                          \
+    const size_t smem = (size_t)(hist_words<NTH, true>() + kCoverCand) * sizeof(uint32_t);   \
+    if ((e = cudaFuncSetAttribute(cover_kernel<NTH>,                                         \
+                                  cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != \
+        cudaSuccess)                                                                         \
+      return e;                                                                              \
+    cover_kernel<NTH><<<grid, NTH, smem, st>>>(P, bf);                                       \
+    return cudaGetLastError();                                                               \
+  }
+  if (units <= 2LL * nsm) MMSHIFT_COVER(512)
+  MMSHIFT_COVER(256)
+#undef MMSHIFT_COVER
 }
 
 cudaError_t launch_topk(const Problem& P, const Buffers& bf, cudaStream_t st, int32_t* out_idx,
                         bool from_scores) {
   int maxT = 0;
   for (int b = 0; b < P.B; ++b) maxT = max(maxT, P.req[b].t_len);
-  const size_t smem = (size_t)(hist_words<NT>() + min(maxT, kMaxStaged)) * sizeof(uint32_t);
-  cudaError_t e = cudaFuncSetAttribute(topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)((hist_words<NT>() + kMaxStaged) * sizeof(uint32_t)));
+  int dev = 0, nsm = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return e;
   dim3 grid(P.Hkv, P.B, P.L);
-  topk_kernel<<<grid, NT, smem, st>>>(P, bf, out_idx, from_scores ? 1 : 0);
-  return cudaGetLastError();
+  const long long units = (long long)grid.x * grid.y * grid.z;
+  const int staged = min(maxT, kMaxStaged);
+#define MMSHIFT_TOPK(NTT)                                                                        \
+  {                                                                                             \
+    const size_t smem = (size_t)(hist_words<NTT, false>() + kTopkCand + staged) * sizeof(uint32_t); \
+    if ((e = cudaFuncSetAttribute(topk_kernel<NTT>, cudaFuncAttributeMaxDynamicSharedMemorySize,  \
+                                  (int)smem)) != cudaSuccess)                                   \
+      return e;                                                                                 \
+    topk_kernel<NTT><<<grid, NTT, smem, st>>>(P, bf, out_idx, from_scores ? 1 : 0, staged);      \
+    return cudaGetLastError();                                                                  \
+  }
+  if (units <= nsm) MMSHIFT_TOPK(1024)
+  MMSHIFT_TOPK(512)
+#undef MMSHIFT_TOPK
 }
 
 cudaError_t launch_gather(const Problem& P, const Buffers& bf, cudaStream_t st, const void* K,
