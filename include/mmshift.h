@@ -134,9 +134,10 @@ typedef struct {
   /* Stage timing: if n_stage_events >= MMSHIFT_N_STAGES + 1, stage_events
    * holds caller-created cudaEvent_t handles and event i is recorded on
    * `stream` just before stage i is enqueued (the last one after the last
-   * stage). Stages: proxies, softmax pass, normaliser merge, mass pass, mass
-   * sum, coverage vote, top-k, gather; a stage that does not run records its
-   * event next to its neighbour's. */
+   * stage). Stages: proxies, softmax pass, normaliser merge, mass pass,
+   * anchor normalisation (tensor-core calls whose anchor rows stay out of the
+   * softmax pass) and mass sum, coverage vote, top-k, gather; a stage that
+   * does not run records its event next to its neighbour's. */
   void** stage_events;
   int32_t n_stage_events;
   int32_t launches;   /* out: number of kernels the call enqueued */

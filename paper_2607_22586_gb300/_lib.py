@@ -63,7 +63,7 @@ class Shape(ctypes.Structure):
 
 
 MMSHIFT_N_STAGES = 8
-STAGES = ("proxies", "softmax_pass", "merge", "mass_pass", "mass_sum", "cover", "topk", "gather")
+STAGES = ("proxies", "softmax_pass", "merge", "mass_pass", "anchor_mass_sum", "cover", "topk", "gather")
 
 
 class Debug(ctypes.Structure):

@@ -129,12 +129,14 @@ mmshift_status build_problem(const mmshift_shape* s, const mmshift_params* p, Pr
 }
 
 struct Layout {
-  size_t status, packed, part, cvals, gmass, anchor, alog, bits, scores, refine, refine_stats, total;
+  size_t status, packed, part, cvals, gmass, anchor, alog, apart, bits, scores, refine, refine_stats, total;
 };
 
 // The anchor rows start a 256-row block of their own: on the tensor-core
 // path the softmax pass leaves them out (Problem::anchor_split).
-bool anchor_spills(const Problem& P) { return P.G > 0 && P.n_group_rows % kRowTile == 0; }
+bool anchor_spills(const Problem& P) {
+  return P.G > 0 && P.n_group_rows % kRowTile == 0 && P.r <= kMaxSplitAnchor;
+}
 
 Layout layout_of(const Problem& P) {
   const size_t esz = P.dtype == MMSHIFT_BF16 ? 2 : 4;
@@ -148,6 +150,7 @@ Layout layout_of(const Problem& P) {
   w.gmass = o;  o += align256(L * P.Hkv * (size_t)P.G * P.total_T * sizeof(float));
   w.anchor = o; o += align256(L * P.Hkv * (size_t)P.total_T * sizeof(float));
   w.alog = o;   o += anchor_spills(P) ? align256(L * P.Hkv * (size_t)P.r * P.total_T * sizeof(float)) : 0;
+  w.apart = o;  o += anchor_spills(P) ? align256(L * P.Hkv * (size_t)P.total_splits * kMaxSplitAnchor * sizeof(float2)) : 0;
   w.bits = o;   o += align256(L * P.Hkv * (size_t)P.G * P.total_words * sizeof(uint32_t));
   w.scores = o; o += align256(L * P.Hkv * (size_t)P.total_T * sizeof(float));
   // count word, the list of proxy elements to recompute in float64, then the
@@ -171,6 +174,7 @@ mmshift_status carve(const Problem& P, void* ws, size_t bytes, Buffers* bf) {
   bf->gmass = reinterpret_cast<float*>(base + w.gmass);
   bf->anchor = reinterpret_cast<float*>(base + w.anchor);
   bf->alog = reinterpret_cast<float*>(base + w.alog);
+  bf->apart = reinterpret_cast<float2*>(base + w.apart);
   bf->bits = reinterpret_cast<uint32_t*>(base + w.bits);
   bf->scores = reinterpret_cast<float*>(base + w.scores);
   bf->refine_count = reinterpret_cast<int*>(base + w.refine);
@@ -241,6 +245,7 @@ mmshift_status run_mass(const Problem& P, const Buffers& bf, const void* K, cons
                  : launch_score_simt(P, bf, st, K, mk.ev);
   if (e != cudaSuccess) return cuda_fail(e);
   if ((e = mk.mark(4)) != cudaSuccess) return cuda_fail(e);
+  if ((e = launch_anchor_split(P, bf, st)) != cudaSuccess) return cuda_fail(e);
   if ((e = launch_mass_sum(P, bf, st)) != cudaSuccess) return cuda_fail(e);
   return MMSHIFT_OK;
 }

@@ -13,6 +13,7 @@ namespace mmshift {
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr int kChunk = 16;       // proxy rows per packing chunk (one group id)
 constexpr int kRowTile = 256;    // proxy rows are padded to a multiple of this
+constexpr int kMaxSplitAnchor = 8;  // anchor_split needs r <= this (one warp per anchor row)
 constexpr int kUmmaPartSlots = 4; // softmax partials per (row, split) of the tensor-core pass
 
 // Status bits the kernels OR into the workspace status word.
@@ -71,6 +72,7 @@ struct Buffers {
   float* gmass;       // [L][Hkv][G][T]
   float* anchor;      // [L][Hkv][T]
   float* alog;        // [L][Hkv][r][T] scaled anchor logits (anchor_split only)
+  float2* apart;      // [L][Hkv][total_splits][kMaxSplitAnchor] their (max, sum) per key split
   uint32_t* bits;     // [L][Hkv][G][total_words] coverage bitmaps
   float* scores;      // [L][Hkv][T]
   float* mass;        // [L][Hkv][T] or null
@@ -199,6 +201,7 @@ bool make_tmap_bf16_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d
                        uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t box1);
 bool tmap_encoder_available();
 int umma_launches(const Problem& P);
+cudaError_t launch_anchor_split(const Problem& P, const Buffers& bf, cudaStream_t st);
 cudaError_t launch_merge(const Problem& P, const Buffers& bf, cudaStream_t st);
 // Attention-mass coverage of the kept set idx from the group masses in bf.
 cudaError_t launch_coverage(const Problem& P, const Buffers& bf, const int32_t* idx, float* cov,

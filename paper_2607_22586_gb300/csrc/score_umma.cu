@@ -500,15 +500,15 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           const int a0 = blk.ng * P.RG;
           if (P.anchor_split) {
             // no normalisers yet: the scaled logits go to alog, row by row
-            // (coalesced along keys), for anchor_norm_kernel
-            float v[16];
-            tmem_ld16(tacc + (uint32_t)a0, v);
+            // (coalesced along keys), for anchor_part_kernel / anchor_final_kernel
+            float v[kMaxSplitAnchor];
+            tmem_ld8(tacc + (uint32_t)a0, v);
             tmem_wait_ld();
             if (valid) {
               float* dst = bf.alog + ((size_t)x.l * P.Hkv + x.h) * P.r * P.total_T + col;
 #pragma unroll
-              for (int j = 0; j < 16; ++j)
-                if (j < P.r) dst[(size_t)j * P.total_T] = v[j] * alpha;
+              for (int a = 0; a < kMaxSplitAnchor; ++a)
+                if (a < P.r) dst[(size_t)a * P.total_T] = v[a] * alpha;
             }
           } else {
             const float sm = group_sum(tacc + (uint32_t)a0, cv + a0, P.anchor_rows, alpha);
@@ -773,41 +773,85 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NTHREADS, 1)
 // ---------------------------------------------------------------- anchor rows (anchor_split)
 // The anchor is the last window query's attention over the request's keys,
 // averaged over the r query heads of the KV head (Section 3.2.3). With
-// anchor_split its logits come from the mass pass (alog, already scaled to
-// log2 units); here, per (KV head, request, layer): c_j = log2 sum_t
-// exp2(y_jt) for each anchor row j, then anchor_t = (sum_j exp2(y_jt - c_j))
-// / r. The reductions run in a fixed order (thread strides, then xor
-// shuffles, then warps in order), so the result does not depend on the other
-// units of the call.
+// anchor_split the mass pass writes its logits (alog, log2 units). Then, per
+// (key split, KV head, layer): anchor_part_kernel takes each anchor row's
+// (max, sum of exp2(y - max)) over the split's keys (apart), and
+// anchor_final_kernel merges the request's partials in split order into c_j =
+// log2 sum_t exp2(y_jt) and writes anchor_t = (sum_j exp2(y_jt - c_j)) / r
+// for the split's keys. All reductions run in a fixed order, so the result
+// does not depend on the other requests or layers of the call.
 constexpr int ANT = 256;
 
-__global__ void __launch_bounds__(ANT) anchor_norm_kernel(const __grid_constant__ Problem P,
+__device__ __forceinline__ int split_request(const Problem& P, int s) {
+  int b = 0;
+  while (b + 1 < P.B && P.req[b + 1].split_off <= s) ++b;
+  return b;
+}
+
+// warp j: anchor row j over the split's keys, 32 keys per round
+__global__ void __launch_bounds__(ANT) anchor_part_kernel(const __grid_constant__ Problem P,
                                                           Buffers bf) {
-  const int h = blockIdx.x, b = blockIdx.y, l = blockIdx.z;
-  const ReqInfo R = P.req[b];
-  const int n = R.t_len, tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
-  const float* y0 = bf.alog + ((size_t)l * P.Hkv + h) * P.r * P.total_T + R.tok_off;
-  __shared__ float wm[ANT / 32][16], wz[ANT / 32][16], cs[16];
-  for (int j = 0; j < P.r; ++j) {
-    const float* y = y0 + (size_t)j * P.total_T;
+  const int s = blockIdx.x, h = blockIdx.y, l = blockIdx.z;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  if (w >= P.r) return;
+  const ReqInfo R = P.req[split_request(P, s)];
+  const int t0 = (s - R.split_off) * P.split_len, t1 = min(R.t_len, t0 + P.split_len);
+  const float* y = bf.alog + (((size_t)l * P.Hkv + h) * P.r + w) * P.total_T + R.tok_off;
+  constexpr int U = 8;
+  float m = -INFINITY, z = 0.f;
+  for (int base = t0; base < t1; base += U * 32) {
+    float v[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int t = base + u * 32 + lane;
+      v[u] = t < t1 ? y[t] : -INFINITY;
+    }
+    float cm = v[0];
+#pragma unroll
+    for (int u = 1; u < U; ++u) cm = fmaxf(cm, v[u]);
+    if (cm == -INFINITY) continue;
+    if (cm > m) {
+      z *= fast_exp2(m - cm);       // 0 while m is still -inf
+      m = cm;
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) z += fast_exp2(v[u] - m);
+  }
+  for (int off = 16; off; off >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+    const float z2 = __shfl_xor_sync(0xffffffffu, z, off);
+    merge_ms(m, z, m2, z2);
+  }
+  if (lane == 0)
+    bf.apart[(((size_t)l * P.Hkv + h) * P.total_splits + s) * kMaxSplitAnchor + w] = make_float2(m, z);
+}
+
+__global__ void __launch_bounds__(ANT) anchor_final_kernel(const __grid_constant__ Problem P,
+                                                           Buffers bf) {
+  const int s = blockIdx.x, h = blockIdx.y, l = blockIdx.z;
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  const ReqInfo R = P.req[split_request(P, s)];
+  const int t0 = (s - R.split_off) * P.split_len, t1 = min(R.t_len, t0 + P.split_len);
+  __shared__ float cs[kMaxSplitAnchor];
+  if (w < P.r) {
+    const float2* src =
+        bf.apart + (((size_t)l * P.Hkv + h) * P.total_splits + R.split_off) * kMaxSplitAnchor + w;
     float m = -INFINITY, z = 0.f;
-    for (int t = tid; t < n; t += ANT) merge_ms(m, z, y[t], 1.f);
+    for (int i = lane; i < R.nsplit; i += 32) {
+      const float2 v = src[(size_t)i * kMaxSplitAnchor];
+      merge_ms(m, z, v.x, v.y);
+    }
     for (int off = 16; off; off >>= 1) {
       const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
       const float z2 = __shfl_xor_sync(0xffffffffu, z, off);
       merge_ms(m, z, m2, z2);
     }
-    if (lane == 0) { wm[w][j] = m; wz[w][j] = z; }
+    if (lane == 0) cs[w] = m + __log2f(z);
   }
   __syncthreads();
-  if (tid < P.r) {
-    float m = -INFINITY, z = 0.f;
-    for (int i = 0; i < ANT / 32; ++i) merge_ms(m, z, wm[i][tid], wz[i][tid]);
-    cs[tid] = m + __log2f(z);
-  }
-  __syncthreads();
+  const float* y0 = bf.alog + ((size_t)l * P.Hkv + h) * P.r * P.total_T + R.tok_off;
   float* out = bf.anchor + ((size_t)l * P.Hkv + h) * P.total_T + R.tok_off;
-  for (int t = tid; t < n; t += ANT) {
+  for (int t = t0 + tid; t < t1; t += ANT) {
     float sm = 0.f;
     for (int j = 0; j < P.r; ++j) sm += fast_exp2(y0[(size_t)j * P.total_T + t] - cs[j]);
     out[t] = sm / (float)P.r;
@@ -901,10 +945,6 @@ cudaError_t launch_d(const Problem& P, const Buffers& bf, cudaStream_t st, const
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
-  if (P.anchor_split && P.total_T) {
-    anchor_norm_kernel<<<dim3(P.Hkv, P.B, P.L), ANT, 0, st>>>(P, bf);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  }
   return cudaSuccess;
 }
 
@@ -950,7 +990,18 @@ bool umma_supported(const Problem& P) {
   return major == 10 && tmap_encoder_available();
 }
 
-int umma_launches(const Problem& P) { return P.anchor_split ? 4 : 3; }
+int umma_launches(const Problem& P) { return P.anchor_split ? 5 : 3; }
+
+// The anchor rows of an anchor_split call, after the mass pass (their own
+// stage, so that the mass pass is timed alone).
+cudaError_t launch_anchor_split(const Problem& P, const Buffers& bf, cudaStream_t st) {
+  if (!P.anchor_split || !P.total_T) return cudaSuccess;
+  anchor_part_kernel<<<dim3(P.total_splits, P.Hkv, P.L), ANT, 0, st>>>(P, bf);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  anchor_final_kernel<<<dim3(P.total_splits, P.Hkv, P.L), ANT, 0, st>>>(P, bf);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_score_umma(const Problem& P, const Buffers& bf, cudaStream_t st,
                               const void* K, cudaEvent_t* ev) {

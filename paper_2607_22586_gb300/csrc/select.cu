@@ -26,7 +26,7 @@ namespace mmshift {
 namespace {
 
 constexpr int kTopkCand = 4096;   // first-digit candidates a top-k CTA keeps in shared memory
-constexpr int kCoverCand = 6144;  // first-digit candidates a coverage CTA keeps in shared memory
+constexpr int kCoverCand = 3072;  // first-digit candidates (key, index) a coverage CTA keeps in shared memory
 constexpr int NBIN = 256;
 constexpr int kMaxStaged = 40960; // top-k keys staged in shared memory (160 KB)
 
@@ -63,13 +63,17 @@ struct SelShared {
   int aux;
 };
 
-// Key source: shared memory when staged, else recomputed from global floats.
-struct KeySrc {
+// Key sources, chosen at compile time: keys staged in shared memory, or
+// recomputed from global floats (read four at a time where aligned).
+struct SmemKeys {
+  static constexpr bool kGlobal = false;
   const uint32_t* smem;
+  __device__ __forceinline__ uint32_t operator()(int i) const { return smem[i]; }
+};
+struct GlobalFloats {
+  static constexpr bool kGlobal = true;
   const float* gmem;
-  __device__ __forceinline__ uint32_t operator()(int i) const {
-    return smem ? smem[i] : nonneg_key(__ldg(gmem + i));
-  }
+  __device__ __forceinline__ uint32_t operator()(int i) const { return nonneg_key(__ldg(gmem + i)); }
 };
 
 // Weight of a key in 2^-shift units: x * 2^shift is exact (a power-of-two
@@ -123,8 +127,8 @@ __device__ __forceinline__ unsigned warp_excl_prefix(SelShared<NTH>& S, unsigned
 // One digit pass: per-warp histograms of the keys matching `prefix` above
 // bit `hs`, digit = bits [sh, hs). Weighted: also the weights, and in the
 // first pass the exact total (returned through S.wsum) and the largest key.
-template <bool WEIGHTED, int NTH>
-__device__ __forceinline__ void digit_histogram(const KeySrc& get, int n, uint32_t prefix, int sh,
+template <bool WEIGHTED, int NTH, class Src>
+__device__ __forceinline__ void digit_histogram(const Src& get, int n, uint32_t prefix, int sh,
                                                 int hs, uint32_t dmask, int shift, bool first,
                                                 SelShared<NTH>& S, uint32_t* hist) {
   constexpr int NWH = NTH / 32;
@@ -154,7 +158,7 @@ __device__ __forceinline__ void digit_histogram(const KeySrc& get, int n, uint32
     }
   };
   int done = 0;
-  if (!get.smem && (reinterpret_cast<uintptr_t>(get.gmem) & 15) == 0) {
+  if constexpr (Src::kGlobal) if ((reinterpret_cast<uintptr_t>(get.gmem) & 15) == 0) {
     // 16-byte loads of four keys, four loads in flight per thread
     constexpr int U4 = 4;
     const float4* g4 = reinterpret_cast<const float4*>(get.gmem);
@@ -269,8 +273,8 @@ __device__ __forceinline__ void digit_scan(unsigned long long target_w, unsigned
 // min(total, ceil(tau * total)) of the exact fixed-point total (S.total) and
 // lowers *shift (redoing the pass) if 2^shift units could overflow 64 bits.
 // `hist` is hist_words<NTH, WEIGHTED>() words of shared memory.
-template <bool WEIGHTED, int NTH>
-__device__ void radix_passes(const KeySrc& get, int n, int p0, int p1, uint32_t& prefix,
+template <bool WEIGHTED, int NTH, class Src>
+__device__ void radix_passes(const Src& get, int n, int p0, int p1, uint32_t& prefix,
                              unsigned long long& target_w, unsigned target_n, int* shift,
                              float tau, SelShared<NTH>& S, uint32_t* hist) {
   constexpr int NWH = NTH / 32;
@@ -282,7 +286,7 @@ __device__ void radix_passes(const KeySrc& get, int n, int p0, int p1, uint32_t&
     const int wid = pass == 3 ? 7 : 8;
     const int sh = pass == 3 ? 0 : 23 - 8 * pass, hs = sh + wid;
     const uint32_t dmask = (1u << wid) - 1u;
-    digit_histogram<WEIGHTED, NTH>(get, n, prefix, sh, hs, dmask, WEIGHTED ? *shift : 0,
+    digit_histogram<WEIGHTED, NTH, Src>(get, n, prefix, sh, hs, dmask, WEIGHTED ? *shift : 0,
                                    pass == 0, S, hist);
     if (WEIGHTED && pass == 0) {
       uint32_t kmax = 0;
@@ -294,7 +298,7 @@ __device__ void radix_passes(const KeySrc& get, int n, int p0, int p1, uint32_t&
       if (e + lg + *shift > 63) {               // n * max * 2^shift could overflow
         *shift = max(0, 63 - e - lg);
         __syncthreads();
-        digit_histogram<WEIGHTED, NTH>(get, n, prefix, sh, hs, dmask, *shift, true, S, hist);
+        digit_histogram<WEIGHTED, NTH, Src>(get, n, prefix, sh, hs, dmask, *shift, true, S, hist);
       }
       unsigned long long total = 0;
       for (int i = 0; i < NWH; ++i) total += S.wsum[i];
@@ -309,12 +313,12 @@ __device__ void radix_passes(const KeySrc& get, int n, int p0, int p1, uint32_t&
   }
 }
 
-template <bool WEIGHTED, int NTH>
-__device__ void radix_select(const KeySrc& get, int n, unsigned long long target_w,
+template <bool WEIGHTED, int NTH, class Src>
+__device__ void radix_select(const Src& get, int n, unsigned long long target_w,
                              unsigned target_n, int* shift, float tau, SelShared<NTH>& S,
                              uint32_t* hist) {
   uint32_t prefix = 0x80000000u;
-  radix_passes<WEIGHTED, NTH>(get, n, 0, 4, prefix, target_w, target_n, shift, tau, S, hist);
+  radix_passes<WEIGHTED, NTH, Src>(get, n, 0, 4, prefix, target_w, target_n, shift, tau, S, hist);
   if (threadIdx.x == 0) S.prefix = prefix;
   __syncthreads();
 }
@@ -324,8 +328,8 @@ __device__ void radix_select(const KeySrc& get, int n, unsigned long long target
 // every thread. Used after the first digit pass, when the keys sharing the
 // chosen first digit fit in shared memory: the later passes then read only
 // them. Each warp appends a ballot's worth at a time.
-template <int NTH>
-__device__ int compact_prefix(const KeySrc& get, int n, uint32_t prefix, int hs, uint32_t* cand,
+template <int NTH, class Src>
+__device__ int compact_prefix(const Src& get, int n, uint32_t prefix, int hs, uint32_t* cand,
                               SelShared<NTH>& S) {
   const int tid = threadIdx.x, lane = tid & 31;
   if (tid == 0) S.ncand = 0;
@@ -342,7 +346,7 @@ __device__ int compact_prefix(const KeySrc& get, int n, uint32_t prefix, int hs,
     if (m) cand[base + __popc(bal & below)] = k;
   };
   int done = 0;
-  if (!get.smem && (reinterpret_cast<uintptr_t>(get.gmem) & 15) == 0) {
+  if constexpr (Src::kGlobal) if ((reinterpret_cast<uintptr_t>(get.gmem) & 15) == 0) {
     constexpr int U4 = 4;
     const float4* g4 = reinterpret_cast<const float4*>(get.gmem);
     const int n4 = n >> 2;
@@ -383,7 +387,7 @@ template <int NTH>
 __global__ void __launch_bounds__(NTH, 1024 / NTH) cover_kernel(Problem P, Buffers bf) {
   extern __shared__ uint32_t dyn[];
   uint32_t* hist = dyn;
-  uint32_t* cand = dyn + hist_words<NTH, true>();   // kCoverCand keys
+  uint32_t* cand = dyn + hist_words<NTH, true>();   // kCoverCand keys, then their indices
   __shared__ SelShared<NTH> S;
   constexpr int NWC = NTH / 32;
   const int g = blockIdx.x % P.G, h = blockIdx.x / P.G, b = blockIdx.y, l = blockIdx.z;
@@ -394,18 +398,73 @@ __global__ void __launch_bounds__(NTH, 1024 / NTH) cover_kernel(Problem P, Buffe
   // the first digit pass reads the masses from L2 / DRAM; when the keys that
   // share the chosen first digit fit in shared memory they are copied there
   // and the last three passes read only them
-  KeySrc get{nullptr, m};
+  const GlobalFloats get{m};
   int shift = 40;
   uint32_t prefix = 0x80000000u;
   unsigned long long target_w = 0;
   radix_passes<true, NTH>(get, n, 0, 1, prefix, target_w, 1u, &shift, P.tau, S, hist);
+  uint32_t* bits = bf.bits + row * P.total_words + R.word_off;
+  constexpr int U = 8;
   if (S.n_theta <= (unsigned)kCoverCand) {
-    const int nc = compact_prefix<NTH>(get, n, prefix, 23, cand, S);
-    radix_passes<true, NTH>(KeySrc{cand, nullptr}, nc, 1, 4, prefix, target_w, 1u, &shift, P.tau,
-                            S, hist);
-  } else {
-    radix_passes<true, NTH>(get, n, 1, 4, prefix, target_w, 1u, &shift, P.tau, S, hist);
+    // One more pass over the masses: keys above the chosen first digit are in
+    // the cover set (their bitmap words are written now), keys sharing it are
+    // copied to shared memory with their indices; the last three digits and
+    // the ties are resolved among those, whose bits are then added.
+    uint32_t* cidx = cand + kCoverCand;
+    if (tid == 0) S.ncand = 0;
+    __syncthreads();
+    const uint32_t d0 = prefix >> 23;
+    const unsigned below = (1u << lane) - 1u;
+    for (int base = w * 32; base < n; base += U * NTH) {
+      uint32_t kk[U];
+#pragma unroll
+      for (int j = 0; j < U; ++j) {
+        const int i = base + j * NTH + lane;
+        kk[j] = i < n ? get(i) : 0u;
+      }
+#pragma unroll
+      for (int j = 0; j < U; ++j) {
+        const int i = base + j * NTH + lane;
+        const bool in = i < n && (kk[j] >> 23) > d0;
+        const bool c = i < n && (kk[j] >> 23) == d0;
+        const unsigned word = __ballot_sync(0xffffffffu, in);
+        if (lane == 0 && base + j * NTH < n) bits[(base + j * NTH) >> 5] = word;
+        const unsigned cb = __ballot_sync(0xffffffffu, c);
+        if (cb) {
+          unsigned at = 0;
+          if (lane == 0) at = atomicAdd(&S.ncand, (unsigned)__popc(cb));
+          at = __shfl_sync(0xffffffffu, at, 0) + __popc(cb & below);
+          if (c) { cand[at] = kk[j]; cidx[at] = (uint32_t)i; }
+        }
+      }
+    }
+    __syncthreads();
+    const int nc = (int)S.ncand;
+    radix_passes<true, NTH>(SmemKeys{cand}, nc, 1, 4, prefix, target_w, 1u, &shift, P.tau, S, hist);
+    const uint32_t theta = prefix;
+    const unsigned n_theta = S.n_theta;
+    const unsigned long long target =
+        min(S.total, (unsigned long long)ceil((double)P.tau * (double)S.total));
+    const unsigned long long wth = fx_weight(theta, pow2f(shift));
+    const unsigned long long need_w = target > S.cum_w ? target - S.cum_w : 0ull;
+    unsigned n_tie = 1;
+    if (need_w > 0 && wth > 0) n_tie = (unsigned)((need_w + wth - 1) / wth);
+    if (n_tie > n_theta) n_tie = n_theta;
+    // a key equal to theta is in if fewer than n_tie equal keys precede it
+    for (int c = tid; c < nc; c += NTH) {
+      const uint32_t k = cand[c], i = cidx[c];
+      bool in = k > theta;
+      if (k == theta) {
+        unsigned rank = 0;
+        if (n_tie < n_theta)
+          for (int e = 0; e < nc; ++e) rank += (cand[e] == theta && cidx[e] < i) ? 1u : 0u;
+        in = rank < n_tie;
+      }
+      if (in) atomicOr(bits + (i >> 5), 1u << (i & 31));
+    }
+    return;
   }
+  radix_passes<true, NTH>(get, n, 1, 4, prefix, target_w, 1u, &shift, P.tau, S, hist);
   if (tid == 0) S.prefix = prefix;
   __syncthreads();
   const uint32_t theta = S.prefix;
@@ -447,8 +506,6 @@ __global__ void __launch_bounds__(NTH, 1024 / NTH) cover_kernel(Problem P, Buffe
   }
   __syncthreads();
   const int tstar = S.aux;
-  uint32_t* bits = bf.bits + row * P.total_words + R.word_off;
-  constexpr int U = 8;
   for (int base = w * 32; base < n; base += U * NTH) {
     uint32_t kk[U];
 #pragma unroll
@@ -464,6 +521,58 @@ __global__ void __launch_bounds__(NTH, 1024 / NTH) cover_kernel(Problem P, Buffe
       if (lane == 0 && base + j * NTH < n) bits[(base + j * NTH) >> 5] = word;
     }
   }
+}
+
+// The keep - 1 largest keys among t < n - 1 (ties: lower t), written to out
+// (stride ostride) in ascending t, then n - 1 last. The first digit is taken
+// over all candidates, the later digits over the keys that share it, copied
+// to shared memory when they fit (cand, kTopkCand keys).
+template <int NT, class Src>
+__device__ void select_kept(const Src& get, int n, int keep, int32_t* out, int ostride,
+                            SelShared<NT>& S, uint32_t* hist, uint32_t* cand) {
+  constexpr int NW = NT / 32;
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  const int nc = n - 1;  // candidates t < T-1
+  uint32_t theta = 0x80000000u;
+  unsigned long long no_w = 0;
+  radix_passes<false, NT, Src>(get, nc, 0, 1, theta, no_w, (unsigned)(keep - 1), nullptr, 0.f, S,
+                               hist);
+  if (S.n_theta <= (unsigned)kTopkCand) {
+    const int ncand = compact_prefix<NT, Src>(get, nc, theta, 23, cand, S);
+    radix_passes<false, NT, SmemKeys>(SmemKeys{cand}, ncand, 1, 4, theta, no_w,
+                                      (unsigned)(keep - 1), nullptr, 0.f, S, hist);
+  } else {
+    radix_passes<false, NT, Src>(get, nc, 1, 4, theta, no_w, (unsigned)(keep - 1), nullptr, 0.f, S,
+                                 hist);
+  }
+  const unsigned n_tie = (unsigned)(keep - 1) - S.cum_n;
+  // ordered compaction over warp segments
+  const int seg = ((nc + NW * 32 - 1) / (NW * 32)) * 32;
+  const int lo = w * seg, hi = min(nc, lo + seg);
+  unsigned c_gt = 0, c_tie = 0;
+  for (int base = lo; base < hi; base += 32) {
+    const int i = base + lane;
+    const uint32_t k = i < hi ? get(i) : 0u;
+    c_gt += __popc(__ballot_sync(0xffffffffu, i < hi && k > theta));
+    c_tie += __popc(__ballot_sync(0xffffffffu, i < hi && k == theta));
+  }
+  const unsigned gt_before = warp_excl_prefix<NT>(S, c_gt);
+  unsigned tie_before = warp_excl_prefix<NT>(S, c_tie);
+  unsigned pos = gt_before + min(tie_before, n_tie);
+  const unsigned lt = (1u << lane) - 1u;
+  for (int base = lo; base < hi; base += 32) {
+    const int i = base + lane;
+    const uint32_t k = i < hi ? get(i) : 0u;
+    const bool is_tie = i < hi && k == theta;
+    const unsigned tie_m = __ballot_sync(0xffffffffu, is_tie);
+    const unsigned my_rank = tie_before + __popc(tie_m & lt);
+    const bool sel = i < hi && (k > theta || (is_tie && my_rank < n_tie));
+    const unsigned sel_m = __ballot_sync(0xffffffffu, sel);
+    if (sel) out[(size_t)(pos + __popc(sel_m & lt)) * ostride] = i;
+    pos += __popc(sel_m);
+    tie_before += __popc(tie_m);
+  }
+  if (tid == 0) out[(size_t)(keep - 1) * ostride] = n - 1;
 }
 
 // from_scores: S comes from bf.scores as given; otherwise it is built here.
@@ -503,16 +612,31 @@ __global__ void __launch_bounds__(NT, 1) topk_kernel(Problem P, Buffers bf, int3
           const int i = base0 + u * NT + lane;
           av[u] = i < n ? __ldg(an + i) : 0.f;
         }
-        for (int g0 = 0; g0 < P.G; g0 += 32) {
-          const int g = g0 + lane;
-          uint32_t word[UB];
+        if (P.G <= 8) {
+          // few groups: every lane reads the chunk's word of each group (one
+          // broadcast load) and takes its own bit
+          for (int g = 0; g < P.G; ++g) {
+            uint32_t word[UB];
 #pragma unroll
-          for (int u = 0; u < UB; ++u) {
-            const int base = base0 + u * NT;
-            word[u] = (g < P.G && base < n) ? __ldg(bw + (size_t)g * P.total_words + (base >> 5)) : 0u;
+            for (int u = 0; u < UB; ++u) {
+              const int base = base0 + u * NT;
+              word[u] = base < n ? __ldg(bw + (size_t)g * P.total_words + (base >> 5)) : 0u;
+            }
+#pragma unroll
+            for (int u = 0; u < UB; ++u) vote[u] += (word[u] >> lane) & 1u;
           }
+        } else {
+          for (int g0 = 0; g0 < P.G; g0 += 32) {
+            const int g = g0 + lane;
+            uint32_t word[UB];
 #pragma unroll
-          for (int u = 0; u < UB; ++u) vote[u] += __popc(warp_transpose32(word[u]));
+            for (int u = 0; u < UB; ++u) {
+              const int base = base0 + u * NT;
+              word[u] = (g < P.G && base < n) ? __ldg(bw + (size_t)g * P.total_words + (base >> 5)) : 0u;
+            }
+#pragma unroll
+            for (int u = 0; u < UB; ++u) vote[u] += __popc(warp_transpose32(word[u]));
+          }
         }
 #pragma unroll
         for (int u = 0; u < UB; ++u)
@@ -563,48 +687,8 @@ __global__ void __launch_bounds__(NT, 1) topk_kernel(Problem P, Buffers bf, int3
     if (tid == 0) out[0] = n - 1;
     return;
   }
-  KeySrc get{staged ? keys_sm : nullptr, sc};
-  const int nc = n - 1;  // candidates t < T-1
-  // first digit over all candidates; the later digits over the keys that
-  // share it, copied to shared memory when they fit
-  uint32_t theta = 0x80000000u;
-  unsigned long long no_w = 0;
-  radix_passes<false, NT>(get, nc, 0, 1, theta, no_w, (unsigned)(keep - 1), nullptr, 0.f, S, hist);
-  if (S.n_theta <= (unsigned)kTopkCand) {
-    const int ncand = compact_prefix<NT>(get, nc, theta, 23, cand, S);
-    radix_passes<false, NT>(KeySrc{cand, nullptr}, ncand, 1, 4, theta, no_w, (unsigned)(keep - 1),
-                            nullptr, 0.f, S, hist);
-  } else {
-    radix_passes<false, NT>(get, nc, 1, 4, theta, no_w, (unsigned)(keep - 1), nullptr, 0.f, S, hist);
-  }
-  const unsigned n_tie = (unsigned)(keep - 1) - S.cum_n;
-  // ordered compaction over warp segments
-  const int seg = ((nc + NW * 32 - 1) / (NW * 32)) * 32;
-  const int lo = w * seg, hi = min(nc, lo + seg);
-  unsigned c_gt = 0, c_tie = 0;
-  for (int base = lo; base < hi; base += 32) {
-    const int i = base + lane;
-    const uint32_t k = i < hi ? get(i) : 0u;
-    c_gt += __popc(__ballot_sync(0xffffffffu, i < hi && k > theta));
-    c_tie += __popc(__ballot_sync(0xffffffffu, i < hi && k == theta));
-  }
-  const unsigned gt_before = warp_excl_prefix<NT>(S, c_gt);
-  unsigned tie_before = warp_excl_prefix<NT>(S, c_tie);
-  unsigned pos = gt_before + min(tie_before, n_tie);
-  const unsigned lt = (1u << lane) - 1u;
-  for (int base = lo; base < hi; base += 32) {
-    const int i = base + lane;
-    const uint32_t k = i < hi ? get(i) : 0u;
-    const bool is_tie = i < hi && k == theta;
-    const unsigned tie_m = __ballot_sync(0xffffffffu, is_tie);
-    const unsigned my_rank = tie_before + __popc(tie_m & lt);
-    const bool sel = i < hi && (k > theta || (is_tie && my_rank < n_tie));
-    const unsigned sel_m = __ballot_sync(0xffffffffu, sel);
-    if (sel) out[(size_t)(pos + __popc(sel_m & lt)) * P.Hkv] = i;
-    pos += __popc(sel_m);
-    tie_before += __popc(tie_m);
-  }
-  if (tid == 0) out[(size_t)(keep - 1) * P.Hkv] = n - 1;
+  if (staged) select_kept<NT>(SmemKeys{keys_sm}, n, keep, out, P.Hkv, S, hist, cand);
+  else select_kept<NT>(GlobalFloats{sc}, n, keep, out, P.Hkv, S, hist, cand);
 }
 
 // mass[l][h][t] = sum over g (ascending) of gmass[l][h][g][t].
@@ -668,7 +752,7 @@ cudaError_t launch_cover(const Problem& P, const Buffers& bf, cudaStream_t st) {
   const long long units = (long long)grid.x * grid.y * grid.z;
 #define MMSHIFT_COVER(NTH)                                                                    \
   {                                                                                          \
-    const size_t smem = (size_t)(hist_words<NTH, true>() + kCoverCand) * sizeof(uint32_t);   \
+    const size_t smem = (size_t)(hist_words<NTH, true>() + 2 * kCoverCand) * sizeof(uint32_t); \
     if ((e = cudaFuncSetAttribute(cover_kernel<NTH>,                                         \
                                   cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != \
         cudaSuccess)                                                                         \
