@@ -59,13 +59,14 @@ METRIC = "prompt tokens selected/sec per layer + % of GB300 HBM roofline (bytes 
 SFU_EX2_PER_SM_CLK = 32          # MUFU.EX2 lanes per SM per clock on GB300 (measured ~31)
 
 # DRAM traffic (read + write) of the two scoring kernels per launch of the
-# default workload: one ncu capture of the full 28-layer workload (the
-# launch-list pass with the two DRAM byte counters, first 16 launches), mean
-# over the two steps captured. It describes only the score_umma.cu it was
-# measured on (checked by hash).
-SCORE_TRAFFIC = {"source_sha256_16": "b46d58a266d0a563", "workload": "qwen7b-28l-32k",
-                 "proxies": "paper", "softmax_pass": 1518.0e6 + 420.7e6,
-                 "mass_pass": 1783.9e6 + 479.9e6}
+# default workload: one ncu capture of a 4-layer slice (the two DRAM byte
+# counters and the duration, one kernel launch each), scaled by 7 to the 28
+# layers (the passes' units grow in proportion to the layers; K read per
+# launch: softmax pass 1.17x, mass pass 1.22x in the slice). It describes
+# only the score_umma.cu it was measured on (checked by hash).
+SCORE_TRAFFIC = {"source_sha256_16": "4b85123b41d48e53", "workload": "qwen7b-28l-32k",
+                 "proxies": "paper", "softmax_pass": 7 * (156.606976e6 + 42.417408e6),
+                 "mass_pass": 7 * (164.298752e6 + 53.264640e6)}
 # DRAM traffic of the prompt-query statistics pass (both kernels) per launch
 # of the default workload, from one ncu capture of a 4-layer slice scaled by 7
 # (partial kernel 939.590912 MB read + 3.059712 MB written, merge 11.026176 MB
