@@ -112,28 +112,45 @@ __global__ void __launch_bounds__(256) pass1_simt(Problem P, Buffers bf, const T
             rt * TILE + row] = make_float2(run_m, run_z);
 }
 
+// Four threads per row: thread q of a row merges the row's partials q, q + 4,
+// q + 8, ... in order (eight loads issued ahead), then the four results are
+// merged by two xor-shuffle steps; the order is fixed, so the result is the
+// same for every launch shape.
+constexpr int kMergeSub = 4;
+
 __global__ void merge_kernel(Problem P, Buffers bf) {
-  const int p = blockIdx.x * blockDim.x + threadIdx.x;
+  const int q = threadIdx.x % kMergeSub;
+  const int p = blockIdx.x * (blockDim.x / kMergeSub) + threadIdx.x / kMergeSub;
   const int bh = blockIdx.y, l = blockIdx.z;
   const int b = bh / P.Hkv, h = bh - b * P.Hkv;
   // with anchor_split the softmax pass has no partials for the anchor rows
-  if (p >= (P.anchor_split ? P.n_group_rows : P.Prows_pad)) return;
+  const int rows = P.anchor_split ? P.n_group_rows : P.Prows_pad;
+  const bool live = p < rows;
   const ReqInfo R = P.req[b];
   float m = -INFINITY, z = 0.f;
-  const float2* src =
-      bf.part + (((size_t)l * P.Hkv + h) * P.total_splits + R.split_off) * P.part_slots * P.Prows_pad + p;
-  // partials merged in split order; eight loads issued ahead of the merges
-  const int ns = R.nsplit * P.part_slots;
+  const float2* src = bf.part +
+                      (((size_t)l * P.Hkv + h) * P.total_splits + R.split_off) * P.part_slots * P.Prows_pad +
+                      (live ? p : 0);
+  const int ns = live ? R.nsplit * P.part_slots : 0;
   constexpr int A = 8;
-  for (int s0 = 0; s0 < ns; s0 += A) {
+  for (int s0 = q; s0 < ns; s0 += A * kMergeSub) {
     float2 v[A];
 #pragma unroll
-    for (int u = 0; u < A; ++u)
-      v[u] = s0 + u < ns ? src[(size_t)(s0 + u) * P.Prows_pad] : make_float2(-INFINITY, 0.f);
+    for (int u = 0; u < A; ++u) {
+      const int si = s0 + u * kMergeSub;
+      v[u] = si < ns ? src[(size_t)si * P.Prows_pad] : make_float2(-INFINITY, 0.f);
+    }
 #pragma unroll
     for (int u = 0; u < A; ++u)
-      if (s0 + u < ns) merge_ms(m, z, v[u].x, v[u].y);
+      if (s0 + u * kMergeSub < ns) merge_ms(m, z, v[u].x, v[u].y);
   }
+#pragma unroll
+  for (int off = 1; off < kMergeSub; off <<= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+    const float z2 = __shfl_xor_sync(0xffffffffu, z, off);
+    merge_ms(m, z, m2, z2);
+  }
+  if (!live || q) return;
   const bool valid = row_kind(P, p).group >= 0;
   bf.cvals[(((size_t)l * P.B + b) * P.Hkv + h) * P.Prows_pad + p] =
       valid ? m + __log2f(z) : INFINITY;
@@ -232,8 +249,10 @@ cudaError_t launch_t(const Problem& P, const Buffers& bf, cudaStream_t st, const
 }  // namespace
 
 cudaError_t launch_merge(const Problem& P, const Buffers& bf, cudaStream_t st) {
-  dim3 grid((P.Prows_pad + 127) / 128, P.B * P.Hkv, P.L);
-  merge_kernel<<<grid, 128, 0, st>>>(P, bf);
+  constexpr int threads = 256, rows_per_block = threads / kMergeSub;
+  const int rows = P.anchor_split ? P.n_group_rows : P.Prows_pad;
+  dim3 grid((rows + rows_per_block - 1) / rows_per_block, P.B * P.Hkv, P.L);
+  merge_kernel<<<grid, threads, 0, st>>>(P, bf);
   return cudaGetLastError();
 }
 

@@ -234,6 +234,32 @@ def test_topk_exact_on_generated_scores(lens, budgets):
                                           O.select_topk(s[hh, lo:hi].astype(np.float64), budgets[b]))
 
 
+@pytest.mark.parametrize("tiny", ["all", "most"])
+def test_topk_exact_with_tiny_scores(tiny):
+    """Scores scaled by 2^-50 (every key, or 80% of them), so that the radix
+    digits fall in the float's low exponents: the kept sets still equal the
+    oracle's."""
+    wl = RAGGED.replace(seq_lens=(5000, 700), n_visual=(0, 0), budgets=(700, 64))
+    T, hkv = wl.total_tokens, wl.n_kv_heads
+    s = S.make_scores(hkv, T, 32, seed=11)
+    rng = np.random.default_rng(3)
+    small = np.ones(s.shape, dtype=bool) if tiny == "all" else rng.random(s.shape) < 0.8
+    s = np.where(small, s * np.float32(2.0 ** -50), s).astype(np.float32)
+    shape = PT.shape_of(wl)
+    ws_bytes = M.mmshift_workspace_size(shape, None)
+    ws = torch.zeros(ws_bytes, dtype=torch.uint8, device="cuda")
+    rows = M.mmshift_output_rows(shape)
+    idx = torch.full((1, rows, hkv), -1, dtype=torch.int32, device="cuda")
+    M.check(M.mmshift_topk(shape, torch.from_numpy(s).cuda(), idx, ws, ws_bytes), "topk")
+    torch.cuda.synchronize()
+    idx = PT.host(idx)[0]
+    for b, lo, hi, olo in _requests(wl):
+        keep = min(wl.budgets[b], hi - lo)
+        for hh in range(hkv):
+            np.testing.assert_array_equal(idx[olo:olo + keep, hh],
+                                          O.select_topk(s[hh, lo:hi].astype(np.float64), wl.budgets[b]))
+
+
 def test_gather_bit_exact_and_bad_index_reported():
     wl = RAGGED
     li = S.make_layer(wl, 1)
