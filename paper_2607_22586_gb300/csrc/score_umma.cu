@@ -269,7 +269,7 @@ __device__ __forceinline__ void mass_chunk(const float (&v)[16], const uint64_t 
   }
 }
 
-// Sum over the ncols (multiple of 16) accumulator columns of one group:
+// Sum over the ncols (multiple of 8) accumulator columns of one group:
 // sum_j exp2(acc_j * alpha - c_j), four partial sums added in a fixed order.
 // nc points at the warp's shared-memory copy of the block's negated normalisers.
 __device__ __forceinline__ float group_sum(uint32_t tcol, const float* nc, int ncols, float alpha) {
@@ -287,13 +287,30 @@ __device__ __forceinline__ float group_sum(uint32_t tcol, const float* nc, int n
     load_nc16(nc + cc + 16, ncv);
     mass_chunk(*reinterpret_cast<float(*)[16]>(v + 16), ncv, al2, a01, a23);
   }
-  if (cc < ncols) {
+  if (cc + 16 <= ncols) {
     float v[16];
     uint64_t ncv[8];
     tmem_ld16(tcol + cc, v);
     load_nc16(nc + cc, ncv);
     tmem_wait_ld();
     mass_chunk(v, ncv, al2, a01, a23);
+    cc += 16;
+  }
+  if (cc < ncols) {   // an 8-column tail (the anchor rows, r <= 8)
+    float v[8];
+    tmem_ld8(tcol + cc, v);
+    const ulonglong2* c2 = reinterpret_cast<const ulonglong2*>(nc + cc);
+    const ulonglong2 n0 = c2[0], n1 = c2[1];
+    tmem_wait_ld();
+    float y0, y1, y2, y3;
+    upk2(ffma2(pk2(v[0], v[1]), al2, n0.x), y0, y1);
+    upk2(ffma2(pk2(v[2], v[3]), al2, n0.y), y2, y3);
+    a01 = fadd2(a01, pk2(fast_exp2(y0), fast_exp2(y1)));
+    a23 = fadd2(a23, pk2(fast_exp2(y2), fast_exp2(y3)));
+    upk2(ffma2(pk2(v[4], v[5]), al2, n1.x), y0, y1);
+    upk2(ffma2(pk2(v[6], v[7]), al2, n1.y), y2, y3);
+    a01 = fadd2(a01, pk2(fast_exp2(y0), fast_exp2(y1)));
+    a23 = fadd2(a23, pk2(fast_exp2(y2), fast_exp2(y3)));
   }
   float a0, a1, a2, a3;
   upk2(a01, a0, a1);
@@ -511,7 +528,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
                 if (a < P.r) dst[(size_t)a * P.total_T] = v[a] * alpha;
             }
           } else {
-            const float sm = group_sum(tacc + (uint32_t)a0, cv + a0, P.anchor_rows, alpha);
+            // the r anchor rows, in 8-column steps (the padding rows up to 16
+            // would add exp2(-inf) = 0)
+            const float sm = group_sum(tacc + (uint32_t)a0, cv + a0, (P.r + 7) & ~7, alpha);
             if (valid)
               bf.anchor[((size_t)x.l * P.Hkv + x.h) * P.total_T + col] = sm / (float)P.r;
           }
