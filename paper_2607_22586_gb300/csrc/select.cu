@@ -127,20 +127,32 @@ __device__ __forceinline__ unsigned warp_excl_prefix(SelShared<NTH>& S, unsigned
 // One digit pass: per-warp histograms of the keys matching `prefix` above
 // bit `hs`, digit = bits [sh, hs). Weighted: also the weights, and in the
 // first pass the exact total (returned through S.wsum) and the largest key.
-template <bool WEIGHTED, int NTH, class Src>
+// ONE: every warp adds into one CTA-wide histogram (for the few candidate
+// keys of the later digits, where combining per-warp copies would cost more
+// than the atomics' contention).
+template <bool WEIGHTED, int NTH, class Src, bool ONE = false>
 __device__ __forceinline__ void digit_histogram(const Src& get, int n, uint32_t prefix, int sh,
                                                 int hs, uint32_t dmask, int shift, bool first,
                                                 SelShared<NTH>& S, uint32_t* hist) {
-  constexpr int NWH = NTH / 32;
+  constexpr int NWH = ONE ? 1 : NTH / 32;
   const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
-  uint32_t* hn = hist + w * NBIN;
-  uint32_t* hlo = hist + (NWH + w) * NBIN;
-  uint32_t* hhi = hist + (2 * NWH + w) * NBIN;
-  for (int i = lane; i < NBIN; i += 32) {
-    hn[i] = 0;
-    if (WEIGHTED) { hlo[i] = 0; hhi[i] = 0; }
+  const int hw = ONE ? 0 : w;
+  uint32_t* hn = hist + hw * NBIN;
+  uint32_t* hlo = hist + (NWH + hw) * NBIN;
+  uint32_t* hhi = hist + (2 * NWH + hw) * NBIN;
+  if (ONE) {
+    for (int i = tid; i < NBIN; i += NTH) {
+      hn[i] = 0;
+      if (WEIGHTED) { hlo[i] = 0; hhi[i] = 0; }
+    }
+    __syncthreads();
+  } else {
+    for (int i = lane; i < NBIN; i += 32) {
+      hn[i] = 0;
+      if (WEIGHTED) { hlo[i] = 0; hhi[i] = 0; }
+    }
+    __syncwarp();
   }
-  __syncwarp();
   unsigned long long tot = 0;
   uint32_t kmax = 0;
   const float scale = pow2f(shift);
@@ -273,7 +285,7 @@ __device__ __forceinline__ void digit_scan(unsigned long long target_w, unsigned
 // min(total, ceil(tau * total)) of the exact fixed-point total (S.total) and
 // lowers *shift (redoing the pass) if 2^shift units could overflow 64 bits.
 // `hist` is hist_words<NTH, WEIGHTED>() words of shared memory.
-template <bool WEIGHTED, int NTH, class Src>
+template <bool WEIGHTED, int NTH, class Src, bool ONE = false>
 __device__ void radix_passes(const Src& get, int n, int p0, int p1, uint32_t& prefix,
                              unsigned long long& target_w, unsigned target_n, int* shift,
                              float tau, SelShared<NTH>& S, uint32_t* hist) {
@@ -286,8 +298,8 @@ __device__ void radix_passes(const Src& get, int n, int p0, int p1, uint32_t& pr
     const int wid = pass == 3 ? 7 : 8;
     const int sh = pass == 3 ? 0 : 23 - 8 * pass, hs = sh + wid;
     const uint32_t dmask = (1u << wid) - 1u;
-    digit_histogram<WEIGHTED, NTH, Src>(get, n, prefix, sh, hs, dmask, WEIGHTED ? *shift : 0,
-                                   pass == 0, S, hist);
+    digit_histogram<WEIGHTED, NTH, Src, ONE>(get, n, prefix, sh, hs, dmask, WEIGHTED ? *shift : 0,
+                                             pass == 0, S, hist);
     if (WEIGHTED && pass == 0) {
       uint32_t kmax = 0;
       for (int i = 0; i < NWH; ++i) kmax = max(kmax, S.wcnt[i]);
@@ -298,7 +310,7 @@ __device__ void radix_passes(const Src& get, int n, int p0, int p1, uint32_t& pr
       if (e + lg + *shift > 63) {               // n * max * 2^shift could overflow
         *shift = max(0, 63 - e - lg);
         __syncthreads();
-        digit_histogram<WEIGHTED, NTH, Src>(get, n, prefix, sh, hs, dmask, *shift, true, S, hist);
+        digit_histogram<WEIGHTED, NTH, Src, ONE>(get, n, prefix, sh, hs, dmask, *shift, true, S, hist);
       }
       unsigned long long total = 0;
       for (int i = 0; i < NWH; ++i) total += S.wsum[i];
@@ -440,7 +452,8 @@ __global__ void __launch_bounds__(NTH, 1024 / NTH) cover_kernel(Problem P, Buffe
     }
     __syncthreads();
     const int nc = (int)S.ncand;
-    radix_passes<true, NTH>(SmemKeys{cand}, nc, 1, 4, prefix, target_w, 1u, &shift, P.tau, S, hist);
+    radix_passes<true, NTH, SmemKeys, true>(SmemKeys{cand}, nc, 1, 4, prefix, target_w, 1u, &shift,
+                                            P.tau, S, hist);
     const uint32_t theta = prefix;
     const unsigned n_theta = S.n_theta;
     const unsigned long long target =
@@ -539,8 +552,8 @@ __device__ void select_kept(const Src& get, int n, int keep, int32_t* out, int o
                                hist);
   if (S.n_theta <= (unsigned)kTopkCand) {
     const int ncand = compact_prefix<NT, Src>(get, nc, theta, 23, cand, S);
-    radix_passes<false, NT, SmemKeys>(SmemKeys{cand}, ncand, 1, 4, theta, no_w,
-                                      (unsigned)(keep - 1), nullptr, 0.f, S, hist);
+    radix_passes<false, NT, SmemKeys, true>(SmemKeys{cand}, ncand, 1, 4, theta, no_w,
+                                            (unsigned)(keep - 1), nullptr, 0.f, S, hist);
   } else {
     radix_passes<false, NT, Src>(get, nc, 1, 4, theta, no_w, (unsigned)(keep - 1), nullptr, 0.f, S,
                                  hist);
@@ -595,10 +608,57 @@ __global__ void __launch_bounds__(NT, 1) topk_kernel(Problem P, Buffers bf, int3
   if (!from_scores) {
     const float* an = bf.anchor + hrow;
     const uint32_t* bw = bf.bits + ((size_t)l * P.Hkv + h) * P.G * P.total_words + R.word_off;
+    int done = 0;
+    if (P.mode == MMSHIFT_SCORE_VOTE && P.G <= 8 && staged &&
+        ((reinterpret_cast<uintptr_t>(an) | reinterpret_cast<uintptr_t>(sc)) & 15) == 0) {
+      // four keys per lane: 16-byte loads of the anchors and stores of the
+      // scores and keys; a lane's keys 4j .. 4j+3 are bits (4j mod 32) .. +3
+      // of coverage word 4j / 32 (one word serves eight lanes)
+      constexpr int UB4 = 4;
+      const float4* an4 = reinterpret_cast<const float4*>(an);
+      float4* sc4 = reinterpret_cast<float4*>(sc);
+      uint4* ks4 = reinterpret_cast<uint4*>(keys_sm);
+      const int n4 = (n >> 5) << 3;   // whole 32-key words only: the rest goes below
+      for (int b4 = w * 32; b4 < n4; b4 += UB4 * NT) {
+        float4 a[UB4];
+        uint32_t vt[UB4];   // four 8-bit vote counters per lane
+#pragma unroll
+        for (int u = 0; u < UB4; ++u) {
+          const int j4 = b4 + u * NT + lane;
+          a[u] = j4 < n4 ? __ldg(an4 + j4) : make_float4(0.f, 0.f, 0.f, 0.f);
+          vt[u] = 0;
+        }
+        for (int g = 0; g < P.G; ++g) {
+#pragma unroll
+          for (int u = 0; u < UB4; ++u) {
+            const int j4 = b4 + u * NT + lane;
+            const uint32_t word =
+                j4 < n4 ? __ldg(bw + (size_t)g * P.total_words + (j4 >> 3)) : 0u;
+            const uint32_t nib = (word >> ((j4 & 7) * 4)) & 0xFu;
+            // spread the nibble's bits into the bytes of vt
+            vt[u] += (nib & 1u) | ((nib & 2u) << 7) | ((nib & 4u) << 14) | ((nib & 8u) << 21);
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < UB4; ++u) {
+          const int j4 = b4 + u * NT + lane;
+          if (j4 < n4) {
+            float4 sv;
+            sv.x = __fadd_rn((float)(vt[u] & 255u), __fmul_rn(P.lambda, a[u].x));
+            sv.y = __fadd_rn((float)((vt[u] >> 8) & 255u), __fmul_rn(P.lambda, a[u].y));
+            sv.z = __fadd_rn((float)((vt[u] >> 16) & 255u), __fmul_rn(P.lambda, a[u].z));
+            sv.w = __fadd_rn((float)(vt[u] >> 24), __fmul_rn(P.lambda, a[u].w));
+            sc4[j4] = sv;
+            ks4[j4] = make_uint4(nonneg_key(sv.x), nonneg_key(sv.y), nonneg_key(sv.z), nonneg_key(sv.w));
+          }
+        }
+      }
+      done = n4 << 2;
+    }
     // each warp takes 32 consecutive keys at a time, UB chunks of them with
-    // their loads in flight together
+    // their loads in flight together (the keys the 16-byte path left, if any)
     constexpr int UB = NT >= 1024 ? 4 : 8;
-    for (int base0 = w * 32; base0 < n; base0 += UB * NT) {
+    for (int base0 = done + w * 32; base0 < n; base0 += UB * NT) {
       float sv[UB];
       if (P.mode == MMSHIFT_SCORE_VOTE) {
         // lane g holds the coverage word of group g for a chunk of 32 keys;
