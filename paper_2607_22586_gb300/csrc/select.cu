@@ -348,14 +348,29 @@ __device__ int compact_prefix(const Src& get, int n, uint32_t prefix, int hs, ui
   __syncthreads();
   const uint32_t want = prefix >> hs;
   const unsigned below = (1u << lane) - 1u;
-  auto put = [&](uint32_t k, bool valid) {
-    const bool m = valid && (k >> hs) == want;
-    const unsigned bal = __ballot_sync(0xffffffffu, m);
-    if (!bal) return;
-    unsigned base = 0;
-    if (lane == 0) base = atomicAdd(&S.ncand, (unsigned)__popc(bal));
-    base = __shfl_sync(0xffffffffu, base, 0);
-    if (m) cand[base + __popc(bal & below)] = k;
+  // a batch of keys per lane: the warp's candidates of the whole batch take
+  // one atomic on the counter, then each key its place from the ballots
+  auto put_batch = [&](const uint32_t* k, const bool* valid, int nb) {
+    unsigned bal[16];
+    unsigned tot = 0;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      if (j < nb) {
+        bal[j] = __ballot_sync(0xffffffffu, valid[j] && (k[j] >> hs) == want);
+        tot += __popc(bal[j]);
+      }
+    }
+    if (!tot) return;
+    unsigned at = 0;
+    if (lane == 0) at = atomicAdd(&S.ncand, tot);
+    at = __shfl_sync(0xffffffffu, at, 0);
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      if (j < nb) {
+        if ((bal[j] >> lane) & 1u) cand[at + __popc(bal[j] & below)] = k[j];
+        at += __popc(bal[j]);
+      }
+    }
   };
   int done = 0;
   if constexpr (Src::kGlobal) if ((reinterpret_cast<uintptr_t>(get.gmem) & 15) == 0) {
@@ -369,27 +384,30 @@ __device__ int compact_prefix(const Src& get, int n, uint32_t prefix, int hs, ui
         const int i4 = base + j * NTH + tid;
         f[j] = i4 < n4 ? __ldg(g4 + i4) : make_float4(0.f, 0.f, 0.f, 0.f);
       }
+      uint32_t kk[4 * U4];
+      bool va[4 * U4];
 #pragma unroll
       for (int j = 0; j < U4; ++j) {
         const bool valid = base + j * NTH + tid < n4;
-        put(nonneg_key(f[j].x), valid);
-        put(nonneg_key(f[j].y), valid);
-        put(nonneg_key(f[j].z), valid);
-        put(nonneg_key(f[j].w), valid);
+        kk[4 * j] = nonneg_key(f[j].x); kk[4 * j + 1] = nonneg_key(f[j].y);
+        kk[4 * j + 2] = nonneg_key(f[j].z); kk[4 * j + 3] = nonneg_key(f[j].w);
+        va[4 * j] = va[4 * j + 1] = va[4 * j + 2] = va[4 * j + 3] = valid;
       }
+      put_batch(kk, va, 4 * U4);
     }
     done = n4 << 2;
   }
   constexpr int U = 8;
   for (int base = done; base < n; base += U * NTH) {
     uint32_t kk[U];
+    bool va[U];
 #pragma unroll
     for (int j = 0; j < U; ++j) {
       const int i = base + j * NTH + tid;
-      kk[j] = i < n ? get(i) : 0u;
+      va[j] = i < n;
+      kk[j] = va[j] ? get(i) : 0u;
     }
-#pragma unroll
-    for (int j = 0; j < U; ++j) put(kk[j], base + j * NTH + tid < n);
+    put_batch(kk, va, U);
   }
   __syncthreads();
   return (int)S.ncand;
@@ -434,19 +452,29 @@ __global__ void __launch_bounds__(NTH, 1024 / NTH) cover_kernel(Problem P, Buffe
         const int i = base + j * NTH + lane;
         kk[j] = i < n ? get(i) : 0u;
       }
+      unsigned cb[U];
+      unsigned tot = 0;
 #pragma unroll
       for (int j = 0; j < U; ++j) {
         const int i = base + j * NTH + lane;
         const bool in = i < n && (kk[j] >> 23) > d0;
-        const bool c = i < n && (kk[j] >> 23) == d0;
         const unsigned word = __ballot_sync(0xffffffffu, in);
         if (lane == 0 && base + j * NTH < n) bits[(base + j * NTH) >> 5] = word;
-        const unsigned cb = __ballot_sync(0xffffffffu, c);
-        if (cb) {
-          unsigned at = 0;
-          if (lane == 0) at = atomicAdd(&S.ncand, (unsigned)__popc(cb));
-          at = __shfl_sync(0xffffffffu, at, 0) + __popc(cb & below);
-          if (c) { cand[at] = kk[j]; cidx[at] = (uint32_t)i; }
+        cb[j] = __ballot_sync(0xffffffffu, i < n && (kk[j] >> 23) == d0);
+        tot += __popc(cb[j]);
+      }
+      if (tot) {   // the batch's candidates: one atomic for the warp
+        unsigned at = 0;
+        if (lane == 0) at = atomicAdd(&S.ncand, tot);
+        at = __shfl_sync(0xffffffffu, at, 0);
+#pragma unroll
+        for (int j = 0; j < U; ++j) {
+          if ((cb[j] >> lane) & 1u) {
+            const unsigned o = at + __popc(cb[j] & below);
+            cand[o] = kk[j];
+            cidx[o] = (uint32_t)(base + j * NTH + lane);
+          }
+          at += __popc(cb[j]);
         }
       }
     }
@@ -559,31 +587,54 @@ __device__ void select_kept(const Src& get, int n, int keep, int32_t* out, int o
                                  hist);
   }
   const unsigned n_tie = (unsigned)(keep - 1) - S.cum_n;
-  // ordered compaction over warp segments
+  // ordered compaction over warp segments, four 32-key chunks' loads at a time
+  constexpr int UC = 4;
   const int seg = ((nc + NW * 32 - 1) / (NW * 32)) * 32;
   const int lo = w * seg, hi = min(nc, lo + seg);
   unsigned c_gt = 0, c_tie = 0;
-  for (int base = lo; base < hi; base += 32) {
-    const int i = base + lane;
-    const uint32_t k = i < hi ? get(i) : 0u;
-    c_gt += __popc(__ballot_sync(0xffffffffu, i < hi && k > theta));
-    c_tie += __popc(__ballot_sync(0xffffffffu, i < hi && k == theta));
+  for (int base = lo; base < hi; base += UC * 32) {
+    uint32_t kk[UC];
+#pragma unroll
+    for (int u = 0; u < UC; ++u) {
+      const int i = base + u * 32 + lane;
+      kk[u] = i < hi ? get(i) : 0u;
+    }
+#pragma unroll
+    for (int u = 0; u < UC; ++u) {
+      const bool in = base + u * 32 + lane < hi;
+      c_gt += __popc(__ballot_sync(0xffffffffu, in && kk[u] > theta));
+      c_tie += __popc(__ballot_sync(0xffffffffu, in && kk[u] == theta));
+    }
   }
-  const unsigned gt_before = warp_excl_prefix<NT>(S, c_gt);
-  unsigned tie_before = warp_excl_prefix<NT>(S, c_tie);
+  // both exclusive prefixes over the warps at once (counts < 2^32 each)
+  if (lane == 0) S.wsum[w] = (unsigned long long)c_gt | ((unsigned long long)c_tie << 32);
+  __syncthreads();
+  unsigned long long before = 0;
+  for (int i = 0; i < w; ++i) before += S.wsum[i];
+  __syncthreads();
+  const unsigned gt_before = (unsigned)before;
+  unsigned tie_before = (unsigned)(before >> 32);
   unsigned pos = gt_before + min(tie_before, n_tie);
   const unsigned lt = (1u << lane) - 1u;
-  for (int base = lo; base < hi; base += 32) {
-    const int i = base + lane;
-    const uint32_t k = i < hi ? get(i) : 0u;
-    const bool is_tie = i < hi && k == theta;
-    const unsigned tie_m = __ballot_sync(0xffffffffu, is_tie);
-    const unsigned my_rank = tie_before + __popc(tie_m & lt);
-    const bool sel = i < hi && (k > theta || (is_tie && my_rank < n_tie));
-    const unsigned sel_m = __ballot_sync(0xffffffffu, sel);
-    if (sel) out[(size_t)(pos + __popc(sel_m & lt)) * ostride] = i;
-    pos += __popc(sel_m);
-    tie_before += __popc(tie_m);
+  for (int base = lo; base < hi; base += UC * 32) {
+    uint32_t kk[UC];
+#pragma unroll
+    for (int u = 0; u < UC; ++u) {
+      const int i = base + u * 32 + lane;
+      kk[u] = i < hi ? get(i) : 0u;
+    }
+#pragma unroll
+    for (int u = 0; u < UC; ++u) {
+      const int i = base + u * 32 + lane;
+      const bool is_tie = i < hi && kk[u] == theta;
+      const unsigned tie_m = __ballot_sync(0xffffffffu, is_tie);
+      const unsigned my_rank = tie_before + __popc(tie_m & lt);
+      const bool sel = i < hi && (kk[u] > theta || (is_tie && my_rank < n_tie));
+      const unsigned sel_m = __ballot_sync(0xffffffffu, sel);
+      if (sel) out[(size_t)(pos + __popc(sel_m & lt)) * ostride] = i;
+      pos += __popc(sel_m);
+      tie_before += __popc(tie_m);
+    }
   }
   if (tid == 0) out[(size_t)(keep - 1) * ostride] = n - 1;
 }
