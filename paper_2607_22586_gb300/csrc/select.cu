@@ -156,6 +156,7 @@ __device__ __forceinline__ void digit_histogram(const Src& get, int n, uint32_t 
   unsigned long long tot = 0;
   uint32_t kmax = 0;
   const float scale = pow2f(shift);
+  const uint32_t wmin = ordered_key(__int_as_float((126 - shift) << 23)) + 1u;
   auto count = [&](uint32_t k, bool valid) {
     const bool take = valid && (k >> hs) == (prefix >> hs);
     if (!first && !__any_sync(0xffffffffu, take)) return;
@@ -163,7 +164,8 @@ __device__ __forceinline__ void digit_histogram(const Src& get, int n, uint32_t 
       const uint32_t d = (k >> sh) & dmask;
       atomicAdd(&hn[d], 1u);
       if (WEIGHTED) {
-        const unsigned long long wt = fx_weight(k, scale);
+        // keys at or below 2^-(shift+1) weigh 0 units: no conversion
+        const unsigned long long wt = k >= wmin ? fx_weight(k, scale) : 0ull;
         if (first) { tot += wt; kmax = max(kmax, k); }
         add_weight(&hlo[d], &hhi[d], wt);
       }
@@ -480,6 +482,48 @@ __global__ void __launch_bounds__(NTH, 1024 / NTH) cover_kernel(Problem P, Buffe
     }
     __syncthreads();
     const int nc = (int)S.ncand;
+    if (nc <= 64) {
+      // Few candidates (the usual case: the bin that completes the cover
+      // holds a few dozen keys): warp 0 ranks them in (key desc, index asc)
+      // order, adds up the exact weights before each, and the cover set's
+      // last key is the first in that order whose inclusive weight, with
+      // the keys above the bin, reaches the target.
+      if (w == 0) {
+        const float sc = pow2f(shift);
+        uint32_t k[2], ix[2];
+        unsigned long long wt[2], before[2] = {0ull, 0ull};
+        unsigned rank[2] = {0u, 0u};
+        bool has[2];
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+          const int c = lane + 32 * q;
+          has[q] = c < nc;
+          k[q] = has[q] ? cand[c] : 0u;
+          ix[q] = has[q] ? cidx[c] : 0xFFFFFFFFu;
+          wt[q] = has[q] ? fx_weight(k[q], sc) : 0ull;
+        }
+        for (int e = 0; e < nc; ++e) {
+          const uint32_t ke = cand[e], ie = cidx[e];
+          const unsigned long long we = fx_weight(ke, sc);
+#pragma unroll
+          for (int q = 0; q < 2; ++q) {
+            const bool pre = ke > k[q] || (ke == k[q] && ie < ix[q]);
+            rank[q] += pre ? 1u : 0u;
+            before[q] += pre ? we : 0ull;
+          }
+        }
+        const unsigned long long above = S.cum_w;
+        unsigned r_end = 0xFFFFFFFFu;
+#pragma unroll
+        for (int q = 0; q < 2; ++q)
+          if (has[q] && above + before[q] + wt[q] >= target_w) r_end = min(r_end, rank[q]);
+        r_end = __reduce_min_sync(0xffffffffu, r_end);
+#pragma unroll
+        for (int q = 0; q < 2; ++q)
+          if (has[q] && rank[q] <= r_end) atomicOr(bits + (ix[q] >> 5), 1u << (ix[q] & 31));
+      }
+      return;
+    }
     radix_passes<true, NTH, SmemKeys, true>(SmemKeys{cand}, nc, 1, 4, prefix, target_w, 1u, &shift,
                                             P.tau, S, hist);
     const uint32_t theta = prefix;
