@@ -64,9 +64,9 @@ SFU_EX2_PER_SM_CLK = 32          # MUFU.EX2 lanes per SM per clock on GB300 (mea
 # layers (the passes' units grow in proportion to the layers; K read per
 # launch: softmax pass 1.17x, mass pass 1.22x in the slice). It describes
 # only the score_umma.cu it was measured on (checked by hash).
-SCORE_TRAFFIC = {"source_sha256_16": "4b85123b41d48e53", "workload": "qwen7b-28l-32k",
-                 "proxies": "paper", "softmax_pass": 7 * (156.606976e6 + 42.417408e6),
-                 "mass_pass": 7 * (164.298752e6 + 53.264640e6)}
+SCORE_TRAFFIC = {"source_sha256_16": "e3fb41b5b8ddbe88", "workload": "qwen7b-28l-32k",
+                 "proxies": "paper", "softmax_pass": 7 * (156.677120e6 + 42.404352e6),
+                 "mass_pass": 7 * (164.203776e6 + 53.250560e6)}
 # DRAM traffic of the prompt-query statistics pass (both kernels) per launch
 # of the default workload, from one ncu capture of a 4-layer slice scaled by 7
 # (partial kernel 939.590912 MB read + 3.059712 MB written, merge 11.026176 MB

@@ -112,12 +112,12 @@ __global__ void __launch_bounds__(256) pass1_simt(Problem P, Buffers bf, const T
             rt * TILE + row] = make_float2(run_m, run_z);
 }
 
-// Four threads per row: thread q of a row merges the row's partials q, q + 4,
-// q + 8, ... in order (eight loads issued ahead), then the four results are
-// merged by two xor-shuffle steps; the order is fixed, so the result is the
-// same for every launch shape.
-constexpr int kMergeSub = 4;
-
+// SUB threads per row (four when a row has at least 128 partials, else one):
+// thread q of a row merges the row's partials q, q + SUB, q + 2 SUB, ... in
+// order (eight loads issued ahead), then the SUB results are merged by xor
+// shuffles; for a given SUB the order is fixed, and SUB depends only on the
+// call's shape.
+template <int kMergeSub>
 __global__ void merge_kernel(Problem P, Buffers bf) {
   const int q = threadIdx.x % kMergeSub;
   const int p = blockIdx.x * (blockDim.x / kMergeSub) + threadIdx.x / kMergeSub;
@@ -249,10 +249,18 @@ cudaError_t launch_t(const Problem& P, const Buffers& bf, cudaStream_t st, const
 }  // namespace
 
 cudaError_t launch_merge(const Problem& P, const Buffers& bf, cudaStream_t st) {
-  constexpr int threads = 256, rows_per_block = threads / kMergeSub;
+  int max_ns = 0;
+  for (int b = 0; b < P.B; ++b) max_ns = max(max_ns, P.req[b].nsplit * P.part_slots);
   const int rows = P.anchor_split ? P.n_group_rows : P.Prows_pad;
-  dim3 grid((rows + rows_per_block - 1) / rows_per_block, P.B * P.Hkv, P.L);
-  merge_kernel<<<grid, threads, 0, st>>>(P, bf);
+  if (max_ns >= 128) {
+    constexpr int threads = 256, rows_per_block = threads / 4;
+    dim3 grid((rows + rows_per_block - 1) / rows_per_block, P.B * P.Hkv, P.L);
+    merge_kernel<4><<<grid, threads, 0, st>>>(P, bf);
+  } else {
+    constexpr int threads = 128;
+    dim3 grid((rows + threads - 1) / threads, P.B * P.Hkv, P.L);
+    merge_kernel<1><<<grid, threads, 0, st>>>(P, bf);
+  }
   return cudaGetLastError();
 }
 
