@@ -213,6 +213,44 @@ def test_scores_topk_exact_on_generated_masses(tau):
                                           O.select_topk(s_exp.astype(np.float64), wl.budgets[b]))
 
 
+@pytest.mark.parametrize("tau", [0.95, 0.5])
+def test_cover_exact_when_the_threshold_bin_is_crowded(tau):
+    """Group 0's masses all share one float exponent ([0.5, 1), on a grid of
+    2^-8 so that many are equal): the coverage vote's first digit leaves
+    9,000 keys in the threshold's bin, more than its shared-memory candidate
+    list holds, so the later digits, the tie scan and the bitmap pass read
+    the masses; group 1 takes the usual path. Votes and kept sets equal the
+    oracle's."""
+    wl = RAGGED.replace(seq_lens=(9000, 300), n_visual=(8000, 280), budgets=(900, 64))
+    h = PT.hyper(n_proxies=32, n_groups=2, tau=tau)
+    T, hkv, G = wl.total_tokens, wl.n_kv_heads, h["n_groups"]
+    gm = S.make_group_masses(hkv, G, T, 112.0, seed=7)
+    rng = np.random.default_rng(9)
+    flat = (np.floor(rng.uniform(0.5, 1.0, size=(hkv, T)) * 256.0) / 256.0).astype(np.float32)
+    gm[:, 0, :] = flat
+    anchor = S.make_scores(hkv, T, 0, seed=8) * np.float32(0.5)
+    shape = PT.shape_of(wl)
+    params = PT.abi_params(h)
+    ws_bytes = M.mmshift_workspace_size(shape, params)
+    ws = torch.zeros(ws_bytes, dtype=torch.uint8, device="cuda")
+    rows = M.mmshift_output_rows(shape)
+    idx = torch.full((1, rows, hkv), -1, dtype=torch.int32, device="cuda")
+    sc = torch.empty((1, hkv, T), device="cuda")
+    st = M.mmshift_scores_topk(shape, params, torch.from_numpy(gm).cuda(),
+                               torch.from_numpy(anchor).cuda(), sc, idx, ws, ws_bytes)
+    M.check(st, "scores_topk")
+    torch.cuda.synchronize()
+    sc, idx = PT.host(sc)[0], PT.host(idx)[0]
+    for b, lo, hi, olo in _requests(wl):
+        keep = min(wl.budgets[b], hi - lo)
+        for hh in range(hkv):
+            v = O.votes(O.cover_sets(gm[hh, :, lo:hi].astype(np.float64), tau))
+            s_exp = (v.astype(np.float32) + np.float32(h["lam"]) * anchor[hh, lo:hi]).astype(np.float32)
+            np.testing.assert_array_equal(sc[hh, lo:hi], s_exp)
+            np.testing.assert_array_equal(idx[olo:olo + keep, hh],
+                                          O.select_topk(s_exp.astype(np.float64), wl.budgets[b]))
+
+
 @pytest.mark.parametrize("lens,budgets", [((5000,), (700,)), ((1, 2, 3, 64, 65), (1, 1, 2, 10, 64)),
                                           ((60000,), (4096,)), ((33, 4097), (32, 4097))])
 def test_topk_exact_on_generated_scores(lens, budgets):
