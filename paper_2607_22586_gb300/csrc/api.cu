@@ -372,6 +372,7 @@ static mmshift_status select_impl(const mmshift_shape* s, const void* K, const v
   }
   const cudaStream_t cs = (cudaStream_t)stream;
   const StageMarks mk = marks_of(dbg, cs);
+  P.cover_hint = (float)(P.r * P.gs);   // the masses below are softmax sums over r * gs rows
   if ((st = run_mass(P, bf, K, Qwin, cs, mk)) != MMSHIFT_OK) return st;
   cudaError_t e = mk.mark(5);
   if (e == cudaSuccess && P.mode == MMSHIFT_SCORE_VOTE) e = launch_cover(P, bf, cs);

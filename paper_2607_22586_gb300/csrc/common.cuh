@@ -58,6 +58,10 @@ struct Problem {
   // leaves them out, the mass pass writes their scaled logits to alog and
   // anchor_norm_kernel normalises them (set per call)
   int32_t anchor_split;
+  // expected total of one group's masses over a request (its proxy rows:
+  // each row's softmax sums to 1) when the coverage vote reads masses this
+  // library computed, else 0 (set per call); only a hint, checked in use
+  float cover_hint;
   int32_t test_stuck_wait; // test only: see mmshift_debug.test_stuck_wait
   ReqInfo req[MMSHIFT_MAX_BATCH];
 };

@@ -60,6 +60,7 @@ struct SelShared {
   unsigned int n_theta;
   unsigned int max_key;
   unsigned int ncand;
+  unsigned int rend;
   int aux;
 };
 
@@ -76,13 +77,24 @@ struct GlobalFloats {
   __device__ __forceinline__ uint32_t operator()(int i) const { return nonneg_key(__ldg(gmem + i)); }
 };
 
-// Weight of a key in 2^-shift units: x * 2^shift is exact (a power-of-two
-// scale of a finite value well inside the float range), then rounded to an
-// integer.
-__device__ __forceinline__ float pow2f(int shift) { return __int_as_float((127 + shift) << 23); }
-__device__ __forceinline__ unsigned long long fx_weight(uint32_t key, float scale) {
-  const float x = fmaxf(key_value(key), 0.f);
-  return __float2ull_rn(x * scale);
+// Weight of a key (of a non-negative float x) in 2^-shift units: x * 2^shift
+// rounded to the nearest integer, ties to even, saturated at 2^64 - 1 (what
+// a float-to-integer conversion of the exact product gives), in integer
+// arithmetic: x = mant * 2^(e - 150) with the 24-bit significand mant, so
+// the weight is mant shifted left by s = e - 150 + shift, or right by -s
+// with the bits shifted out rounding it.
+__device__ __forceinline__ unsigned long long fx_weight(uint32_t key, int shift) {
+  const uint32_t u = key & 0x7FFFFFFFu;
+  const int e = (int)(u >> 23);
+  const uint32_t mant = (u & 0x7FFFFFu) | 0x800000u;
+  const int s = e - 150 + shift;
+  if (e == 0) return 0ull;                    // zero and subnormals (below 2^-126)
+  if (e == 255 || s > 40) return ~0ull;       // at least 2^64, infinity, NaN
+  if (s >= 0) return (unsigned long long)mant << s;
+  if (s < -24) return 0ull;                   // below one half
+  const int r = -s;                           // 1 .. 24
+  const uint32_t q = mant >> r, rem = mant & ((1u << r) - 1u), half = 1u << (r - 1);
+  return q + ((rem > half || (rem == half && (q & 1u))) ? 1u : 0u);
 }
 
 // Add a 64-bit weight to a histogram bin held as two 32-bit words (low,
@@ -155,7 +167,6 @@ __device__ __forceinline__ void digit_histogram(const Src& get, int n, uint32_t 
   }
   unsigned long long tot = 0;
   uint32_t kmax = 0;
-  const float scale = pow2f(shift);
   const uint32_t wmin = ordered_key(__int_as_float((126 - shift) << 23)) + 1u;
   auto count = [&](uint32_t k, bool valid) {
     const bool take = valid && (k >> hs) == (prefix >> hs);
@@ -165,7 +176,7 @@ __device__ __forceinline__ void digit_histogram(const Src& get, int n, uint32_t 
       atomicAdd(&hn[d], 1u);
       if (WEIGHTED) {
         // keys at or below 2^-(shift+1) weigh 0 units: no conversion
-        const unsigned long long wt = k >= wmin ? fx_weight(k, scale) : 0ull;
+        const unsigned long long wt = k >= wmin ? fx_weight(k, shift) : 0ull;
         if (first) { tot += wt; kmax = max(kmax, k); }
         add_weight(&hlo[d], &hhi[d], wt);
       }
@@ -285,12 +296,14 @@ __device__ __forceinline__ void digit_scan(unsigned long long target_w, unsigned
 // the number of keys that share the chosen first digit (the only keys the
 // later passes look at). Weighted mode: pass 0 sets target_w to
 // min(total, ceil(tau * total)) of the exact fixed-point total (S.total) and
-// lowers *shift (redoing the pass) if 2^shift units could overflow 64 bits.
+// lowers *shift (redoing the pass) if 2^shift units could overflow 64 bits,
+// unless pass0_total is false (target_w and *shift then stand as given).
 // `hist` is hist_words<NTH, WEIGHTED>() words of shared memory.
 template <bool WEIGHTED, int NTH, class Src, bool ONE = false>
 __device__ void radix_passes(const Src& get, int n, int p0, int p1, uint32_t& prefix,
                              unsigned long long& target_w, unsigned target_n, int* shift,
-                             float tau, SelShared<NTH>& S, uint32_t* hist) {
+                             float tau, SelShared<NTH>& S, uint32_t* hist,
+                             bool pass0_total = true) {
   constexpr int NWH = NTH / 32;
   const int tid = threadIdx.x;
   if (p0 == 0 && tid == 0) { S.cum_w = 0; S.cum_n = 0; }
@@ -302,7 +315,7 @@ __device__ void radix_passes(const Src& get, int n, int p0, int p1, uint32_t& pr
     const uint32_t dmask = (1u << wid) - 1u;
     digit_histogram<WEIGHTED, NTH, Src, ONE>(get, n, prefix, sh, hs, dmask, WEIGHTED ? *shift : 0,
                                              pass == 0, S, hist);
-    if (WEIGHTED && pass == 0) {
+    if (WEIGHTED && pass == 0 && pass0_total) {
       uint32_t kmax = 0;
       for (int i = 0; i < NWH; ++i) kmax = max(kmax, S.wcnt[i]);
       int e = 0;
@@ -415,34 +428,348 @@ __device__ int compact_prefix(const Src& get, int n, uint32_t prefix, int hs, ui
   return (int)S.ncand;
 }
 
+// Per-thread asynchronous 16-byte copies global -> shared (completion waited
+// for by the issuing thread with cp.async.wait_group).
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                   (uint32_t)__cvta_generic_to_shared(smem)),
+               "l"(gmem)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// Stages of the shared-memory ring of a streaming pass: NTH quads each, so
+// the ring is exactly the size of the weighted per-warp histograms it
+// shares memory with.
+constexpr int kRingStages = 6;
+static_assert(hist_words<512, true>() * 4 == kRingStages * 512 * 16 &&
+                  hist_words<256, true>() * 4 == kRingStages * 256 * 16,
+              "the streaming ring fills the weighted histograms exactly");
+
+// One pass over m[0, n): the exact total weight (2^-shift units) and the
+// largest key, returned to every thread, and the keys at or above kspec
+// with their indices appended to (cand, cidx) (S.ncand, 0 on entry, counts
+// them all; only the first cap are stored; kspec = ~0 appends none).
+// The quads after a scalar head up to the first 16-byte boundary stream
+// through `ring` (kRingStages * NTH quads of shared memory): thread t
+// copies quads t, t + NTH, ... with cp.async, kRingStages ahead, and reads
+// back only its own copies, so no barrier is needed between the stages.
+template <int NTH>
+__device__ void total_and_max(const float* m, int n, int shift, uint32_t kspec, uint32_t* cand,
+                              uint32_t* cidx, int cap, float4* ring, SelShared<NTH>& S,
+                              unsigned long long& total, uint32_t& kmax) {
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  // keys at or below 2^-(shift+1) weigh 0 units: no conversion
+  const uint32_t wmin = ordered_key(__int_as_float((126 - shift) << 23)) + 1u;
+  unsigned long long tot = 0;
+  uint32_t km = 0;
+  auto append = [&](uint32_t k, int i) {
+    const unsigned o = atomicAdd(&S.ncand, 1u);
+    if (o < (unsigned)cap) { cand[o] = k; cidx[o] = (uint32_t)i; }
+  };
+  auto add1 = [&](float x, int i) {
+    const uint32_t k = nonneg_key(x);
+    km = max(km, k);
+    if (k >= wmin) tot += fx_weight(k, shift);
+    if (k >= kspec) append(k, i);
+  };
+  const int head = min(n, (int)(((16u - (uint32_t)(reinterpret_cast<uintptr_t>(m) & 15)) & 15u) >> 2));
+  if (tid < head) add1(__ldg(m + tid), tid);
+  const float4* g4 = reinterpret_cast<const float4*>(m + head);
+  const int n4 = (n - head) >> 2;
+#pragma unroll
+  for (int s = 0; s < kRingStages; ++s) {
+    const int i4 = s * NTH + tid;
+    if (i4 < n4) cp_async16(ring + s * NTH + tid, g4 + i4);
+    cp_async_commit();
+  }
+  int slot = 0;
+  for (int c = 0; c * NTH < n4; ++c) {
+    cp_async_wait<kRingStages - 1>();
+    const int i4 = c * NTH + tid;
+    if (i4 < n4) {
+      const float4 f = ring[slot * NTH + tid];
+      const uint32_t k0 = nonneg_key(f.x), k1 = nonneg_key(f.y), k2 = nonneg_key(f.z),
+                     k3 = nonneg_key(f.w);
+      km = max(max(km, max(k0, k1)), max(k2, k3));
+      const unsigned long long w0 = k0 >= wmin ? fx_weight(k0, shift) : 0ull;
+      const unsigned long long w1 = k1 >= wmin ? fx_weight(k1, shift) : 0ull;
+      const unsigned long long w2 = k2 >= wmin ? fx_weight(k2, shift) : 0ull;
+      const unsigned long long w3 = k3 >= wmin ? fx_weight(k3, shift) : 0ull;
+      tot += (w0 + w1) + (w2 + w3);
+      if (max(max(k0, k1), max(k2, k3)) >= kspec) {   // rare
+        const int i0 = head + 4 * i4;
+        if (k0 >= kspec) append(k0, i0);
+        if (k1 >= kspec) append(k1, i0 + 1);
+        if (k2 >= kspec) append(k2, i0 + 2);
+        if (k3 >= kspec) append(k3, i0 + 3);
+      }
+    }
+    // the quad this thread just read is in registers: its slot takes the
+    // copy kRingStages chunks ahead
+    const int nx = (c + kRingStages) * NTH + tid;
+    if (nx < n4) cp_async16(ring + slot * NTH + tid, g4 + nx);
+    cp_async_commit();
+    if (++slot == kRingStages) slot = 0;
+  }
+  cp_async_wait<0>();
+  for (int i = head + (n4 << 2) + tid; i < n; i += NTH) add1(__ldg(m + i), i);
+  for (int off = 16; off; off >>= 1) {
+    tot += __shfl_xor_sync(0xffffffffu, tot, off);
+    km = max(km, __shfl_xor_sync(0xffffffffu, km, off));
+  }
+  if (lane == 0) { S.wsum[w] = tot; S.wcnt[w] = km; }
+  __syncthreads();
+  total = 0;
+  kmax = 0;
+  for (int i = 0; i < NTH / 32; ++i) { total += S.wsum[i]; kmax = max(kmax, S.wcnt[i]); }
+  __syncthreads();
+}
+
+// Smallest key (of a non-negative float) whose weight in 2^-shift units is
+// at least wt >= 1 (weights do not decrease with the key).
+__device__ __forceinline__ uint32_t key_of_weight(unsigned long long wt, int shift) {
+  uint32_t lo = 0x80000001u, hi = 0xFF7FFFFFu;   // the largest finite float weighs >= 2^63
+  while (lo < hi) {
+    const uint32_t mid = lo + ((hi - lo) >> 1);
+    if (fx_weight(mid, shift) >= wt) hi = mid; else lo = mid + 1u;
+  }
+  return lo;
+}
+
+// Appends the keys of m[0, n) at or above klb (> the key of 0) with their
+// indices to (cand, cidx), in no particular order, and returns their number
+// to every thread (also when it exceeds cap: only the first cap are kept).
+// S.ncand must be 0 on entry. Each warp takes one atomic per batch of loads.
+template <int NTH>
+__device__ int compact_above(const float* m, int n, uint32_t klb, uint32_t* cand, uint32_t* cidx,
+                             int cap, SelShared<NTH>& S) {
+  const int tid = threadIdx.x, lane = tid & 31;
+  const unsigned below = (1u << lane) - 1u;
+  const int head = min(n, (int)(((16u - (uint32_t)(reinterpret_cast<uintptr_t>(m) & 15)) & 15u) >> 2));
+  const float4* g4 = reinterpret_cast<const float4*>(m + head);
+  const int n4 = (n - head) >> 2;
+  constexpr int U4 = 4;
+  for (int base = 0; base < n4; base += U4 * NTH) {   // the same trip count in every warp
+    float4 f[U4];
+#pragma unroll
+    for (int j = 0; j < U4; ++j) {
+      const int i4 = base + j * NTH + tid;
+      f[j] = i4 < n4 ? __ldg(g4 + i4) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    uint32_t kk[4 * U4];
+    unsigned bal[4 * U4];
+    unsigned tot = 0;
+#pragma unroll
+    for (int j = 0; j < U4; ++j) {
+      kk[4 * j] = nonneg_key(f[j].x); kk[4 * j + 1] = nonneg_key(f[j].y);
+      kk[4 * j + 2] = nonneg_key(f[j].z); kk[4 * j + 3] = nonneg_key(f[j].w);
+    }
+#pragma unroll
+    for (int j = 0; j < 4 * U4; ++j) {
+      bal[j] = __ballot_sync(0xffffffffu, kk[j] >= klb);
+      tot += __popc(bal[j]);
+    }
+    if (!tot) continue;   // the usual case: one atomic per warp and batch otherwise
+    unsigned at = 0;
+    if (lane == 0) at = atomicAdd(&S.ncand, tot);
+    at = __shfl_sync(0xffffffffu, at, 0);
+#pragma unroll
+    for (int j = 0; j < 4 * U4; ++j) {
+      if ((bal[j] >> lane) & 1u) {
+        const unsigned o = at + __popc(bal[j] & below);
+        if (o < (unsigned)cap) {
+          cand[o] = kk[j];
+          cidx[o] = (uint32_t)(head + 4 * (base + (j >> 2) * NTH + tid) + (j & 3));
+        }
+      }
+      at += __popc(bal[j]);
+    }
+  }
+  if (tid < 32) {  // the head and the tail: at most 3 + 3 keys, warp 0
+    const int tail0 = head + (n4 << 2);
+    const int i = tid < head ? tid : tail0 + (tid - 3);
+    const bool has = tid < head || (tid >= 3 && tid < 6 && i < n);
+    const bool in = has && nonneg_key(__ldg(m + i)) >= klb;
+    const unsigned bl = __ballot_sync(0xffffffffu, in);
+    if (bl) {
+      unsigned at = 0;
+      if (lane == 0) at = atomicAdd(&S.ncand, __popc(bl));
+      at = __shfl_sync(0xffffffffu, at, 0) + __popc(bl & below);
+      if (in && at < (unsigned)cap) { cand[at] = nonneg_key(__ldg(m + i)); cidx[at] = (uint32_t)i; }
+    }
+  }
+  __syncthreads();
+  return (int)S.ncand;
+}
+
+// The cover set's keys among the candidates (cand, cidx)[0, nc): every key
+// ranked before them in (key desc, index asc) order weighs S.cum_w in all,
+// every key ranked after them is below all of them, and the last digits
+// from p0 on are still open (prefix holds the chosen ones). The set is the
+// shortest prefix of that order whose weight reaches target_w; its bits are
+// ORed into the bitmap. Up to NTH candidates: each thread ranks one against
+// all the others. More: the remaining digit passes among them, then the
+// keys equal to the last key theta by index.
+template <int NTH>
+__device__ void cover_among(const uint32_t* cand, const uint32_t* cidx, int nc, int p0,
+                            uint32_t prefix, unsigned long long target_w, int shift, float tau,
+                            SelShared<NTH>& S, uint32_t* hist, uint32_t* bits) {
+  const int tid = threadIdx.x;
+  if (nc <= NTH) {
+    // (key << 32 | ~index, weight) per candidate: a larger first word ranks
+    // earlier
+    ulonglong2* cw = reinterpret_cast<ulonglong2*>(hist);
+    if (tid == 0) S.rend = 0xFFFFFFFFu;
+    if (tid < nc)
+      cw[tid] = make_ulonglong2(((unsigned long long)cand[tid] << 32) | (uint32_t)~cidx[tid],
+                                fx_weight(cand[tid], shift));
+    __syncthreads();
+    const unsigned long long above = S.cum_w;
+    unsigned rank = 0;
+    unsigned long long me = 0;
+    if (tid < nc) {
+      const ulonglong2 x = cw[tid];
+      me = x.x;
+      unsigned long long before = 0;
+      int e = 0;
+      for (; e + 4 <= nc; e += 4) {
+        const ulonglong2 y0 = cw[e], y1 = cw[e + 1], y2 = cw[e + 2], y3 = cw[e + 3];
+        rank += (y0.x > me) + (y1.x > me) + (y2.x > me) + (y3.x > me);
+        before += (y0.x > me ? y0.y : 0ull) + (y1.x > me ? y1.y : 0ull) +
+                  (y2.x > me ? y2.y : 0ull) + (y3.x > me ? y3.y : 0ull);
+      }
+      for (; e < nc; ++e) {
+        const ulonglong2 y = cw[e];
+        rank += y.x > me;
+        before += y.x > me ? y.y : 0ull;
+      }
+      if (above + before + x.y >= target_w) atomicMin(&S.rend, rank);
+    }
+    __syncthreads();
+    if (tid < nc && rank <= S.rend) {
+      const uint32_t ix = ~(uint32_t)me;
+      atomicOr(bits + (ix >> 5), 1u << (ix & 31));
+    }
+    return;
+  }
+  radix_passes<true, NTH, SmemKeys, true>(SmemKeys{cand}, nc, p0, 4, prefix, target_w, 1u, &shift,
+                                          tau, S, hist, false);
+  const uint32_t theta = prefix;
+  const unsigned n_theta = S.n_theta;
+  const unsigned long long wth = fx_weight(theta, shift);
+  const unsigned long long need_w = target_w > S.cum_w ? target_w - S.cum_w : 0ull;
+  unsigned n_tie = 1;
+  if (need_w > 0 && wth > 0) n_tie = (unsigned)((need_w + wth - 1) / wth);
+  if (n_tie > n_theta) n_tie = n_theta;
+  // a key equal to theta is in if fewer than n_tie equal keys precede it
+  for (int c = tid; c < nc; c += NTH) {
+    const uint32_t k = cand[c], i = cidx[c];
+    bool in = k > theta;
+    if (k == theta) {
+      unsigned rank = 0;
+      if (n_tie < n_theta)
+        for (int e = 0; e < nc; ++e) rank += (cand[e] == theta && cidx[e] < i) ? 1u : 0u;
+      in = rank < n_tie;
+    }
+    if (in) atomicOr(bits + (i >> 5), 1u << (i & 31));
+  }
+}
+
 template <int NTH>
 __global__ void __launch_bounds__(NTH, 1024 / NTH) cover_kernel(Problem P, Buffers bf) {
   extern __shared__ uint32_t dyn[];
   uint32_t* hist = dyn;
   uint32_t* cand = dyn + hist_words<NTH, true>();   // kCoverCand keys, then their indices
+  uint32_t* cidx = cand + kCoverCand;
   __shared__ SelShared<NTH> S;
   constexpr int NWC = NTH / 32;
   const int g = blockIdx.x % P.G, h = blockIdx.x / P.G, b = blockIdx.y, l = blockIdx.z;
   const ReqInfo R = P.req[b];
   const int n = R.t_len, tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  if (n <= 0) return;
   const size_t row = ((size_t)l * P.Hkv + h) * P.G + g;
   const float* m = bf.gmass + row * P.total_T + R.tok_off;
-  // the first digit pass reads the masses from L2 / DRAM; when the keys that
-  // share the chosen first digit fit in shared memory they are copied there
-  // and the last three passes read only them
-  const GlobalFloats get{m};
-  int shift = 40;
-  uint32_t prefix = 0x80000000u;
-  unsigned long long target_w = 0;
-  radix_passes<true, NTH>(get, n, 0, 1, prefix, target_w, 1u, &shift, P.tau, S, hist);
   uint32_t* bits = bf.bits + row * P.total_words + R.word_off;
+  const GlobalFloats get{m};
+
+  // Only keys of weight >= lb can be in the cover set or tie with its last
+  // key theta, where lb = (total - target + 1) / n: the keys ranked before
+  // theta weigh at most target - 1 (else the cover would end earlier) and
+  // the at most n - 1 after it at most w_theta each, so total <= target - 1
+  // + n * w_theta. With few such keys the cover is decided among them
+  // alone, every other bit being 0. When the masses are softmax sums of a
+  // known number of rows (P.cover_hint), the keys above half the bound that
+  // total implies are collected in the same pass as the total; the
+  // collection stands if its bound is at most lb, else a second pass
+  // collects the keys of weight >= lb.
+  int shift = 40;
+  unsigned long long gspec = 0;
+  if (P.cover_hint > 0.f) {
+    const double g = ((1.0 - (double)P.tau) * 0.5 * (double)P.cover_hint * 1099511627776.0 - 1.0) /
+                     (double)n;                       // 2^40 units
+    gspec = g >= 1.0 ? (unsigned long long)g : 0ull;
+  }
+  if (tid == 0) {
+    S.prefix = gspec ? key_of_weight(gspec, shift) : 0xFFFFFFFFu;
+    S.ncand = 0;
+    S.cum_w = 0;
+    S.cum_n = 0;
+  }
+  for (int i = tid; i < (n + 31) / 32; i += NTH) bits[i] = 0u;
+  __syncthreads();
+  unsigned long long total = 0;
+  uint32_t kmax = 0;
+  total_and_max<NTH>(m, n, shift, S.prefix, cand, cidx, kCoverCand,
+                     reinterpret_cast<float4*>(hist), S, total, kmax);
+  int nc = (int)S.ncand;
+  {
+    // the 2^-shift unit is lowered where n * max * 2^shift could overflow 64 bits
+    int e = 0;
+    frexpf(key_value(kmax), &e);              // values < 2^e
+    int lg = 0;
+    while ((1 << lg) < n) ++lg;               // n <= 2^lg
+    if (e + lg + shift > 63) {
+      shift = max(0, 63 - e - lg);
+      gspec = 0;
+      total_and_max<NTH>(m, n, shift, 0xFFFFFFFFu, cand, cidx, kCoverCand,
+                         reinterpret_cast<float4*>(hist), S, total, kmax);
+    }
+  }
+  const unsigned long long tt = (unsigned long long)ceil((double)P.tau * (double)total);
+  unsigned long long target_w = tt > total ? total : tt;
+  const unsigned long long lb = (total - target_w + 1) / (unsigned long long)n;
+  if (lb > 0) {
+    if (!(gspec > 0 && gspec <= lb && nc <= kCoverCand)) {
+      __syncthreads();   // every thread has read S.ncand
+      if (tid == 0) {
+        S.prefix = key_of_weight(lb, shift);
+        S.ncand = 0;
+      }
+      __syncthreads();
+      nc = compact_above<NTH>(m, n, S.prefix, cand, cidx, kCoverCand, S);
+    }
+    if (nc > 0 && nc <= kCoverCand) {
+      cover_among<NTH>(cand, cidx, nc, 0, 0x80000000u, target_w, shift, P.tau, S, hist, bits);
+      return;
+    }
+  }
+
+  // Many keys above the bound: the first digit pass over the masses (from
+  // L2), then, when the keys that share the chosen first digit fit in shared
+  // memory, one more pass writes the bitmap words of the keys above that
+  // digit and copies the keys sharing it; the last three digits and the ties
+  // are resolved among those.
+  uint32_t prefix = 0x80000000u;
+  radix_passes<true, NTH>(get, n, 0, 1, prefix, target_w, 1u, &shift, P.tau, S, hist);
   constexpr int U = 8;
   if (S.n_theta <= (unsigned)kCoverCand) {
-    // One more pass over the masses: keys above the chosen first digit are in
-    // the cover set (their bitmap words are written now), keys sharing it are
-    // copied to shared memory with their indices; the last three digits and
-    // the ties are resolved among those, whose bits are then added.
-    uint32_t* cidx = cand + kCoverCand;
     if (tid == 0) S.ncand = 0;
     __syncthreads();
     const uint32_t d0 = prefix >> 23;
@@ -481,72 +808,7 @@ __global__ void __launch_bounds__(NTH, 1024 / NTH) cover_kernel(Problem P, Buffe
       }
     }
     __syncthreads();
-    const int nc = (int)S.ncand;
-    if (nc <= 64) {
-      // Few candidates (the usual case: the bin that completes the cover
-      // holds a few dozen keys): warp 0 ranks them in (key desc, index asc)
-      // order, adds up the exact weights before each, and the cover set's
-      // last key is the first in that order whose inclusive weight, with
-      // the keys above the bin, reaches the target.
-      if (w == 0) {
-        const float sc = pow2f(shift);
-        uint32_t k[2], ix[2];
-        unsigned long long wt[2], before[2] = {0ull, 0ull};
-        unsigned rank[2] = {0u, 0u};
-        bool has[2];
-#pragma unroll
-        for (int q = 0; q < 2; ++q) {
-          const int c = lane + 32 * q;
-          has[q] = c < nc;
-          k[q] = has[q] ? cand[c] : 0u;
-          ix[q] = has[q] ? cidx[c] : 0xFFFFFFFFu;
-          wt[q] = has[q] ? fx_weight(k[q], sc) : 0ull;
-        }
-        for (int e = 0; e < nc; ++e) {
-          const uint32_t ke = cand[e], ie = cidx[e];
-          const unsigned long long we = fx_weight(ke, sc);
-#pragma unroll
-          for (int q = 0; q < 2; ++q) {
-            const bool pre = ke > k[q] || (ke == k[q] && ie < ix[q]);
-            rank[q] += pre ? 1u : 0u;
-            before[q] += pre ? we : 0ull;
-          }
-        }
-        const unsigned long long above = S.cum_w;
-        unsigned r_end = 0xFFFFFFFFu;
-#pragma unroll
-        for (int q = 0; q < 2; ++q)
-          if (has[q] && above + before[q] + wt[q] >= target_w) r_end = min(r_end, rank[q]);
-        r_end = __reduce_min_sync(0xffffffffu, r_end);
-#pragma unroll
-        for (int q = 0; q < 2; ++q)
-          if (has[q] && rank[q] <= r_end) atomicOr(bits + (ix[q] >> 5), 1u << (ix[q] & 31));
-      }
-      return;
-    }
-    radix_passes<true, NTH, SmemKeys, true>(SmemKeys{cand}, nc, 1, 4, prefix, target_w, 1u, &shift,
-                                            P.tau, S, hist);
-    const uint32_t theta = prefix;
-    const unsigned n_theta = S.n_theta;
-    const unsigned long long target =
-        min(S.total, (unsigned long long)ceil((double)P.tau * (double)S.total));
-    const unsigned long long wth = fx_weight(theta, pow2f(shift));
-    const unsigned long long need_w = target > S.cum_w ? target - S.cum_w : 0ull;
-    unsigned n_tie = 1;
-    if (need_w > 0 && wth > 0) n_tie = (unsigned)((need_w + wth - 1) / wth);
-    if (n_tie > n_theta) n_tie = n_theta;
-    // a key equal to theta is in if fewer than n_tie equal keys precede it
-    for (int c = tid; c < nc; c += NTH) {
-      const uint32_t k = cand[c], i = cidx[c];
-      bool in = k > theta;
-      if (k == theta) {
-        unsigned rank = 0;
-        if (n_tie < n_theta)
-          for (int e = 0; e < nc; ++e) rank += (cand[e] == theta && cidx[e] < i) ? 1u : 0u;
-        in = rank < n_tie;
-      }
-      if (in) atomicOr(bits + (i >> 5), 1u << (i & 31));
-    }
+    cover_among<NTH>(cand, cidx, (int)S.ncand, 1, prefix, target_w, shift, P.tau, S, hist, bits);
     return;
   }
   radix_passes<true, NTH>(get, n, 1, 4, prefix, target_w, 1u, &shift, P.tau, S, hist);
@@ -554,10 +816,8 @@ __global__ void __launch_bounds__(NTH, 1024 / NTH) cover_kernel(Problem P, Buffe
   __syncthreads();
   const uint32_t theta = S.prefix;
   const unsigned n_theta = S.n_theta;
-  const unsigned long long target =
-      min(S.total, (unsigned long long)ceil((double)P.tau * (double)S.total));
-  const unsigned long long wth = fx_weight(theta, pow2f(shift));
-  const unsigned long long need_w = target > S.cum_w ? target - S.cum_w : 0ull;
+  const unsigned long long wth = fx_weight(theta, shift);
+  const unsigned long long need_w = target_w > S.cum_w ? target_w - S.cum_w : 0ull;
   unsigned n_tie = 1;
   if (need_w > 0 && wth > 0) n_tie = (unsigned)((need_w + wth - 1) / wth);
   if (n_tie > n_theta) n_tie = n_theta;

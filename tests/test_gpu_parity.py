@@ -214,19 +214,27 @@ def test_scores_topk_exact_on_generated_masses(tau):
 
 
 @pytest.mark.parametrize("tau", [0.95, 0.5])
-def test_cover_exact_when_the_threshold_bin_is_crowded(tau):
-    """Group 0's masses all share one float exponent ([0.5, 1), on a grid of
-    2^-8 so that many are equal): the coverage vote's first digit leaves
-    9,000 keys in the threshold's bin, more than its shared-memory candidate
-    list holds, so the later digits, the tie scan and the bitmap pass read
-    the masses; group 1 takes the usual path. Votes and kept sets equal the
-    oracle's."""
+@pytest.mark.parametrize("kind", ["flat", "two_level"])
+def test_cover_exact_when_many_keys_are_heavy(tau, kind):
+    """Group 0's masses make the coverage vote leave its usual path (a few
+    keys above the bound on the last cover key's weight, ranked one per
+    thread). flat: all masses share one float exponent ([0.5, 1), on a grid
+    of 2^-8 so that many are equal), so every key is above the bound and
+    9,000 share the threshold's first digit, more than the shared-memory
+    candidate list holds: the digit passes, the tie scan and the bitmap pass
+    read the masses. two_level: 2,000 such keys among light ones (2^-20),
+    more than one per thread but few enough for the list: the digit passes
+    and the tie ranking run among them. Group 1 takes the usual path. Votes
+    and kept sets equal the oracle's."""
     wl = RAGGED.replace(seq_lens=(9000, 300), n_visual=(8000, 280), budgets=(900, 64))
     h = PT.hyper(n_proxies=32, n_groups=2, tau=tau)
     T, hkv, G = wl.total_tokens, wl.n_kv_heads, h["n_groups"]
     gm = S.make_group_masses(hkv, G, T, 112.0, seed=7)
     rng = np.random.default_rng(9)
     flat = (np.floor(rng.uniform(0.5, 1.0, size=(hkv, T)) * 256.0) / 256.0).astype(np.float32)
+    if kind == "two_level":
+        light = rng.random(size=(hkv, T)) >= 2000.0 / 9000.0
+        flat[light] = np.float32(2.0 ** -20)
     gm[:, 0, :] = flat
     anchor = S.make_scores(hkv, T, 0, seed=8) * np.float32(0.5)
     shape = PT.shape_of(wl)
