@@ -943,10 +943,216 @@ __device__ void select_kept(const Src& get, int n, int keep, int32_t* out, int o
   if (tid == 0) out[(size_t)(keep - 1) * ostride] = n - 1;
 }
 
+// The keep - 1 largest of the staged keys[0, n - 1) (ties: lower t), written
+// to out (stride ostride) in ascending t, then n - 1 last, with a 12-bit
+// first digit (the exponent and the top four significand bits): one
+// CTA-wide histogram of 4096 bins (hist_built: already counted over keys
+// [0, n - 1) by the caller), a block scan for the digit d0 where the
+// count from the top reaches keep - 1, the keys of digit d0 copied to shared
+// memory with their indices and the kept ones among them marked in a bitmap
+// (ranked one per thread when few, else by the last three digit passes and
+// the ties' indices), then one pass over the keys that builds the kept words
+// and a block scan that places them. Returns false (before writing any
+// output) when more than kFineCand keys share d0.
+constexpr int kFineCand = 1024;
+template <int NT>
+__device__ bool select_kept_fine(const uint32_t* keys, int n, int keep, int32_t* out, int ostride,
+                                 SelShared<NT>& S, uint32_t* hist, uint32_t* cand,
+                                 bool hist_built) {
+  constexpr int NW = NT / 32;
+  constexpr int BPT = 4096 / NT;                       // histogram bins per thread
+  constexpr int WPL = (kMaxStaged / (NW * 32) + 31) / 32 + 1;   // kept words per lane
+  static_assert(hist_words<NT, false>() >= 4096, "12-bit histogram in the per-warp histograms' room");
+  static_assert(2 * kFineCand + kMaxStaged / 32 <= kTopkCand, "candidates and kept bits in cand");
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  const int nc = n - 1;                 // candidates t < n - 1
+  const unsigned k = (unsigned)(keep - 1);   // 1 <= k < nc
+  uint32_t* ck = cand;                  // keys of digit d0
+  uint32_t* ci = cand + kFineCand;      // their indices
+  uint32_t* kbits = cand + 2 * kFineCand;    // kept keys of digit d0, by index
+  const int nwords = (nc + 31) >> 5;
+  if (!hist_built) {
+    for (int i = tid; i < 4096; i += NT) hist[i] = 0u;
+    __syncthreads();
+    for (int i = tid; i < nc; i += NT) atomicAdd(&hist[(keys[i] >> 19) & 0xFFFu], 1u);
+  }
+  for (int i = tid; i < nwords; i += NT) kbits[i] = 0u;
+  if (tid == 0) S.ncand = 0;
+  __syncthreads();
+  // thread t owns digits 4095 - BPT t down to 4096 - BPT (t + 1): inclusive
+  // scan of their counts in thread order is the count from the top
+  unsigned c = 0;
+#pragma unroll
+  for (int j = 0; j < BPT; ++j) c += hist[4095 - BPT * tid - j];
+  unsigned incl = c;
+  for (int off = 1; off < 32; off <<= 1) {
+    const unsigned t = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += t;
+  }
+  if (lane == 31) S.wcnt[w] = incl;
+  __syncthreads();
+  for (int i = 0; i < w; ++i) incl += S.wcnt[i];
+  const unsigned excl = incl - c;
+  if (excl < k && incl >= k) {
+    unsigned cum = excl;
+    for (int j = 0; j < BPT; ++j) {
+      const int d = 4095 - BPT * tid - j;
+      const unsigned b = hist[d];
+      if (cum + b >= k) {
+        S.digit = (unsigned)d;
+        S.cum_n = cum;
+        S.n_theta = b;
+        break;
+      }
+      cum += b;
+    }
+  }
+  __syncthreads();
+  const uint32_t d0 = S.digit;
+  const unsigned above = S.cum_n, nd = S.n_theta;
+  if (nd > (unsigned)kFineCand) {
+    __syncthreads();   // every thread has read S before the caller's select rewrites it
+    return false;
+  }
+  // the keys of digit d0 with their indices; a warp's 32 consecutive keys,
+  // four chunks at a time, take one atomic
+  const unsigned below = (1u << lane) - 1u;
+  for (int base = w * 128; base < nc; base += NT * 4) {
+    bool in[4];
+    unsigned bal[4], tot = 0;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int i = base + 32 * u + lane;
+      in[u] = i < nc && ((keys[i] >> 19) & 0xFFFu) == d0;
+      bal[u] = __ballot_sync(0xffffffffu, in[u]);
+      tot += __popc(bal[u]);
+    }
+    if (!tot) continue;
+    unsigned at = 0;
+    if (lane == 0) at = atomicAdd(&S.ncand, tot);
+    at = __shfl_sync(0xffffffffu, at, 0);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (in[u]) {
+        const unsigned o = at + __popc(bal[u] & below);
+        const int i = base + 32 * u + lane;
+        ck[o] = keys[i];
+        ci[o] = (uint32_t)i;
+      }
+      at += __popc(bal[u]);
+    }
+  }
+  __syncthreads();
+  const unsigned need = k - above;      // kept keys of digit d0, 1 <= need <= nd
+  if (nd <= (unsigned)NT) {
+    // (key << 32 | ~index) ranks earlier when larger
+    unsigned long long* comp = reinterpret_cast<unsigned long long*>(hist);
+    if (tid < (int)nd) comp[tid] = ((unsigned long long)ck[tid] << 32) | (uint32_t)~ci[tid];
+    __syncthreads();
+    if (tid < (int)nd) {
+      const unsigned long long me = comp[tid];
+      unsigned rank = 0;
+      int e = 0;
+      for (; e + 4 <= (int)nd; e += 4)
+        rank += (comp[e] > me) + (comp[e + 1] > me) + (comp[e + 2] > me) + (comp[e + 3] > me);
+      for (; e < (int)nd; ++e) rank += comp[e] > me;
+      if (rank < need) {
+        const uint32_t i = ~(uint32_t)me;
+        atomicOr(&kbits[i >> 5], 1u << (i & 31));
+      }
+    }
+  } else {
+    uint32_t theta = ck[0] & 0xFFF80000u;   // bits 19-31 are d0's
+    unsigned long long no_w = 0;
+    radix_passes<false, NT, SmemKeys, true>(SmemKeys{ck}, (int)nd, 1, 4, theta, no_w, k, nullptr,
+                                            0.f, S, hist);
+    const unsigned n_tie = k - S.cum_n;   // keys equal to theta kept, lowest indices first
+    for (int c2 = tid; c2 < (int)nd; c2 += NT) {
+      const uint32_t kk = ck[c2], i = ci[c2];
+      bool kept = kk > theta;
+      if (kk == theta) {
+        unsigned r = 0;
+        for (int e = 0; e < (int)nd; ++e) r += (ck[e] == theta && ci[e] < i) ? 1u : 0u;
+        kept = r < n_tie;
+      }
+      if (kept) atomicOr(&kbits[i >> 5], 1u << (i & 31));
+    }
+  }
+  __syncthreads();
+  // kept words: warp w owns words [w0, w0 + wpw); lane j of row q holds word
+  // w0 + 32 q + j; four words' keys are loaded before their ballots
+  const int wpw = (nwords + NW - 1) / NW;
+  const int w0 = w * wpw;
+  const int nww = max(0, min(wpw, nwords - w0));   // words of this warp
+  uint32_t word[WPL];
+  unsigned row_tot[WPL], row_excl[WPL];
+  unsigned wtot = 0;
+#pragma unroll
+  for (int q = 0; q < WPL; ++q) {
+    word[q] = 0u;
+    const int jn = min(32, nww - 32 * q);   // warp-uniform
+    for (int j0 = 0; j0 < jn; j0 += 4) {
+      uint32_t kk[4];
+      bool ok[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = (w0 + 32 * q + j0 + u) * 32 + lane;
+        ok[u] = j0 + u < jn && i < nc;
+        kk[u] = ok[u] ? keys[i] : 0u;
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = (w0 + 32 * q + j0 + u) * 32 + lane;
+        const uint32_t d = (kk[u] >> 19) & 0xFFFu;
+        const bool kept =
+            ok[u] && (d > d0 || (d == d0 && ((kbits[i >> 5] >> (i & 31)) & 1u)));
+        const unsigned b = __ballot_sync(0xffffffffu, kept);
+        if (lane == j0 + u) word[q] = b;
+      }
+    }
+    const unsigned cnt = __popc(word[q]);
+    unsigned inc = cnt;
+    for (int off = 1; off < 32; off <<= 1) {
+      const unsigned t = __shfl_up_sync(0xffffffffu, inc, off);
+      if (lane >= off) inc += t;
+    }
+    row_excl[q] = inc - cnt;
+    row_tot[q] = __shfl_sync(0xffffffffu, inc, 31);
+    wtot += row_tot[q];
+  }
+  if (lane == 0) S.wcnt[w] = wtot;
+  __syncthreads();
+  unsigned pos = 0;
+  for (int i = 0; i < w; ++i) pos += S.wcnt[i];
+  // the kept indices go to shared memory (the histograms' room) in order,
+  // then out in one coalesced sweep; directly when they do not fit
+  int32_t* staging = reinterpret_cast<int32_t*>(hist);
+  const bool via_smem = k <= (unsigned)hist_words<NT, false>();
+#pragma unroll
+  for (int q = 0; q < WPL; ++q) {
+    unsigned p = pos + row_excl[q];
+    uint32_t m = word[q];
+    const int i0 = (w0 + 32 * q + lane) * 32;
+    while (m) {
+      const int bit = __ffs(m) - 1;
+      m &= m - 1u;
+      if (via_smem) staging[p++] = i0 + bit;
+      else out[(size_t)(p++) * ostride] = i0 + bit;
+    }
+    pos += row_tot[q];
+  }
+  if (via_smem) {
+    __syncthreads();
+    for (int i = tid; i < (int)k; i += NT) out[(size_t)i * ostride] = staging[i];
+  }
+  if (tid == 0) out[(size_t)(keep - 1) * ostride] = n - 1;
+  return true;
+}
+
 // from_scores: S comes from bf.scores as given; otherwise it is built here.
 // NT threads per CTA (512, or 1024 when the units are fewer than the SMs).
 template <int NT>
-__global__ void __launch_bounds__(NT, 1) topk_kernel(Problem P, Buffers bf, int32_t* out_idx,
+__global__ void __launch_bounds__(NT, NT >= 1024 ? 1 : 2) topk_kernel(Problem P, Buffers bf, int32_t* out_idx,
                                                      int from_scores, int staged_cap) {
   constexpr int NW = NT / 32;
   extern __shared__ uint32_t dyn[];
@@ -960,6 +1166,15 @@ __global__ void __launch_bounds__(NT, 1) topk_kernel(Problem P, Buffers bf, int3
   const size_t hrow = ((size_t)l * P.Hkv + h) * P.total_T + R.tok_off;
   float* sc = bf.scores + hrow;
   const bool staged = n <= staged_cap;
+  // staged keys are counted by their 12-bit first digit as they are written
+  // (select_kept_fine), the last key excepted
+  if (staged) {
+    for (int i = tid; i < 4096; i += NT) hist[i] = 0u;
+    __syncthreads();
+  }
+  auto count12 = [&](uint32_t key, int i) {
+    if (i < n - 1) atomicAdd(&hist[(key >> 19) & 0xFFFu], 1u);
+  };
   if (!from_scores) {
     const float* an = bf.anchor + hrow;
     const uint32_t* bw = bf.bits + ((size_t)l * P.Hkv + h) * P.G * P.total_words + R.word_off;
@@ -1004,7 +1219,11 @@ __global__ void __launch_bounds__(NT, 1) topk_kernel(Problem P, Buffers bf, int3
             sv.z = __fadd_rn((float)((vt[u] >> 16) & 255u), __fmul_rn(P.lambda, a[u].z));
             sv.w = __fadd_rn((float)(vt[u] >> 24), __fmul_rn(P.lambda, a[u].w));
             sc4[j4] = sv;
-            ks4[j4] = make_uint4(nonneg_key(sv.x), nonneg_key(sv.y), nonneg_key(sv.z), nonneg_key(sv.w));
+            const uint4 kq = make_uint4(nonneg_key(sv.x), nonneg_key(sv.y), nonneg_key(sv.z),
+                                        nonneg_key(sv.w));
+            ks4[j4] = kq;
+            count12(kq.x, 4 * j4); count12(kq.y, 4 * j4 + 1);
+            count12(kq.z, 4 * j4 + 2); count12(kq.w, 4 * j4 + 3);
           }
         }
       }
@@ -1073,12 +1292,20 @@ __global__ void __launch_bounds__(NT, 1) topk_kernel(Problem P, Buffers bf, int3
         const int i = base0 + u * NT + lane;
         if (i < n) {
           sc[i] = sv[u];
-          if (staged) keys_sm[i] = nonneg_key(sv[u]);
+          if (staged) {
+            const uint32_t kq = nonneg_key(sv[u]);
+            keys_sm[i] = kq;
+            count12(kq, i);
+          }
         }
       }
     }
   } else if (staged) {
-    for (int i = tid; i < n; i += NT) keys_sm[i] = nonneg_key(sc[i]);
+    for (int i = tid; i < n; i += NT) {
+      const uint32_t kq = nonneg_key(sc[i]);
+      keys_sm[i] = kq;
+      count12(kq, i);
+    }
   }
   __syncthreads();
   int32_t* out = out_idx + ((size_t)l * P.R + R.out_off) * P.Hkv + h;
@@ -1102,8 +1329,13 @@ __global__ void __launch_bounds__(NT, 1) topk_kernel(Problem P, Buffers bf, int3
     if (tid == 0) out[0] = n - 1;
     return;
   }
-  if (staged) select_kept<NT>(SmemKeys{keys_sm}, n, keep, out, P.Hkv, S, hist, cand);
-  else select_kept<NT>(GlobalFloats{sc}, n, keep, out, P.Hkv, S, hist, cand);
+  if (staged) {
+    if (!select_kept_fine<NT>(keys_sm, n, keep, out, P.Hkv, S, hist, cand, true))
+      select_kept<NT>(SmemKeys{keys_sm}, n, keep, out, P.Hkv, S, hist, cand);
+  }
+  else {
+    select_kept<NT>(GlobalFloats{sc}, n, keep, out, P.Hkv, S, hist, cand);
+  }
 }
 
 // mass[l][h][t] = sum over g (ascending) of gmass[l][h][g][t].

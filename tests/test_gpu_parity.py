@@ -306,6 +306,33 @@ def test_topk_exact_with_tiny_scores(tiny):
                                           O.select_topk(s[hh, lo:hi].astype(np.float64), wl.budgets[b]))
 
 
+def test_topk_exact_when_the_fine_bin_holds_many_keys():
+    """48 layers x 4 heads, more units than SMs (512-thread CTAs), and per
+    head 20% of 4,000 keys in one 12-bit first-digit bin (scores on a 2^-12
+    grid in [1, 1.0625), so many tie) above keys in [0.25, 0.5): the bin's
+    kept keys are found by the later digit passes and, among equal keys, by
+    index. Kept sets equal the oracle's."""
+    L = 48
+    wl = RAGGED.replace(seq_lens=(4000,), n_visual=(0,), budgets=(300,))
+    T, hkv = wl.total_tokens, wl.n_kv_heads
+    rng = np.random.default_rng(21)
+    s = rng.uniform(0.25, 0.5, size=(L, hkv, T)).astype(np.float32)
+    grid = (1.0 + np.floor(rng.uniform(0.0, 1.0, size=(L, hkv, T)) * 256.0) / 4096.0)
+    s = np.where(rng.random(size=(L, hkv, T)) < 0.2, grid, s).astype(np.float32)
+    shape = PT.shape_of(wl, L)
+    ws_bytes = M.mmshift_workspace_size(shape, None)
+    ws = torch.zeros(ws_bytes, dtype=torch.uint8, device="cuda")
+    rows = M.mmshift_output_rows(shape)
+    idx = torch.full((L, rows, hkv), -1, dtype=torch.int32, device="cuda")
+    M.check(M.mmshift_topk(shape, torch.from_numpy(s).cuda(), idx, ws, ws_bytes), "topk")
+    torch.cuda.synchronize()
+    idx = PT.host(idx)
+    for l in range(L):
+        for hh in range(hkv):
+            np.testing.assert_array_equal(idx[l, :300, hh],
+                                          O.select_topk(s[l, hh].astype(np.float64), 300))
+
+
 def test_gather_bit_exact_and_bad_index_reported():
     wl = RAGGED
     li = S.make_layer(wl, 1)
