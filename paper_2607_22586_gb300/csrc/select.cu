@@ -949,10 +949,10 @@ __device__ void select_kept(const Src& get, int n, int keep, int32_t* out, int o
 // CTA-wide histogram of 4096 bins (hist_built: already counted over keys
 // [0, n - 1) by the caller), a block scan for the digit d0 where the
 // count from the top reaches keep - 1, the keys of digit d0 copied to shared
-// memory with their indices and the kept ones among them marked in a bitmap
-// (ranked one per thread when few, else by the last three digit passes and
-// the ties' indices), then one pass over the keys that builds the kept words
-// and a block scan that places them. Returns false (before writing any
+// memory with their indices while the bitmap of the keys above d0 is
+// written, the kept ones among them added to it (ranked one per thread when
+// few, else by the last three digit passes and the ties' indices), then a
+// block scan over the bitmap's words places the kept indices. Returns false (before writing any
 // output) when more than kFineCand keys share d0.
 constexpr int kFineCand = 1024;
 template <int NT>
@@ -976,7 +976,6 @@ __device__ bool select_kept_fine(const uint32_t* keys, int n, int keep, int32_t*
     __syncthreads();
     for (int i = tid; i < nc; i += NT) atomicAdd(&hist[(keys[i] >> 19) & 0xFFFu], 1u);
   }
-  for (int i = tid; i < nwords; i += NT) kbits[i] = 0u;
   if (tid == 0) S.ncand = 0;
   __syncthreads();
   // thread t owns digits 4095 - BPT t down to 4096 - BPT (t + 1): inclusive
@@ -1014,8 +1013,9 @@ __device__ bool select_kept_fine(const uint32_t* keys, int n, int keep, int32_t*
     __syncthreads();   // every thread has read S before the caller's select rewrites it
     return false;
   }
-  // the keys of digit d0 with their indices; a warp's 32 consecutive keys,
-  // four chunks at a time, take one atomic
+  // the keys of digit d0 with their indices, and the kept-bitmap words of
+  // the keys above d0 (every word of [0, nc) is written here); a warp's 32
+  // consecutive keys, four chunks at a time, take one atomic
   const unsigned below = (1u << lane) - 1u;
   for (int base = w * 128; base < nc; base += NT * 4) {
     bool in[4];
@@ -1023,9 +1023,12 @@ __device__ bool select_kept_fine(const uint32_t* keys, int n, int keep, int32_t*
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       const int i = base + 32 * u + lane;
-      in[u] = i < nc && ((keys[i] >> 19) & 0xFFFu) == d0;
+      const uint32_t d = i < nc ? (keys[i] >> 19) & 0xFFFu : 0u;
+      in[u] = i < nc && d == d0;
       bal[u] = __ballot_sync(0xffffffffu, in[u]);
       tot += __popc(bal[u]);
+      const unsigned gt = __ballot_sync(0xffffffffu, i < nc && d > d0);
+      if (lane == 0 && base + 32 * u < nc) kbits[(base + 32 * u) >> 5] = gt;
     }
     if (!tot) continue;
     unsigned at = 0;
@@ -1079,8 +1082,8 @@ __device__ bool select_kept_fine(const uint32_t* keys, int n, int keep, int32_t*
     }
   }
   __syncthreads();
-  // kept words: warp w owns words [w0, w0 + wpw); lane j of row q holds word
-  // w0 + 32 q + j; four words' keys are loaded before their ballots
+  // kept words (the bitmap above): warp w owns words [w0, w0 + wpw); lane j
+  // of row q holds word w0 + 32 q + j
   const int wpw = (nwords + NW - 1) / NW;
   const int w0 = w * wpw;
   const int nww = max(0, min(wpw, nwords - w0));   // words of this warp
@@ -1089,27 +1092,8 @@ __device__ bool select_kept_fine(const uint32_t* keys, int n, int keep, int32_t*
   unsigned wtot = 0;
 #pragma unroll
   for (int q = 0; q < WPL; ++q) {
-    word[q] = 0u;
-    const int jn = min(32, nww - 32 * q);   // warp-uniform
-    for (int j0 = 0; j0 < jn; j0 += 4) {
-      uint32_t kk[4];
-      bool ok[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int i = (w0 + 32 * q + j0 + u) * 32 + lane;
-        ok[u] = j0 + u < jn && i < nc;
-        kk[u] = ok[u] ? keys[i] : 0u;
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int i = (w0 + 32 * q + j0 + u) * 32 + lane;
-        const uint32_t d = (kk[u] >> 19) & 0xFFFu;
-        const bool kept =
-            ok[u] && (d > d0 || (d == d0 && ((kbits[i >> 5] >> (i & 31)) & 1u)));
-        const unsigned b = __ballot_sync(0xffffffffu, kept);
-        if (lane == j0 + u) word[q] = b;
-      }
-    }
+    const int wi = 32 * q + lane;
+    word[q] = wi < nww ? kbits[w0 + wi] : 0u;
     const unsigned cnt = __popc(word[q]);
     unsigned inc = cnt;
     for (int off = 1; off < 32; off <<= 1) {
