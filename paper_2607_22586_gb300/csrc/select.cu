@@ -80,21 +80,21 @@ struct GlobalFloats {
 // Weight of a key (of a non-negative float x) in 2^-shift units: x * 2^shift
 // rounded to the nearest integer, ties to even, saturated at 2^64 - 1 (what
 // a float-to-integer conversion of the exact product gives), in integer
-// arithmetic: x = mant * 2^(e - 150) with the 24-bit significand mant, so
-// the weight is mant shifted left by s = e - 150 + shift, or right by -s
-// with the bits shifted out rounding it.
+// arithmetic without branches: x = mant * 2^(e - 150) with the 24-bit
+// significand mant, so the weight is mant shifted left by s = e - 150 +
+// shift, or right by r = -s as (mant + 2^(r-1) - 1 + (bit r of mant)) >> r,
+// which rounds half to even (r >= 25 gives 0; r is clamped to 31, which
+// also makes zero and the subnormals weigh 0).
 __device__ __forceinline__ unsigned long long fx_weight(uint32_t key, int shift) {
   const uint32_t u = key & 0x7FFFFFFFu;
   const int e = (int)(u >> 23);
   const uint32_t mant = (u & 0x7FFFFFu) | 0x800000u;
   const int s = e - 150 + shift;
-  if (e == 0) return 0ull;                    // zero and subnormals (below 2^-126)
-  if (e == 255 || s > 40) return ~0ull;       // at least 2^64, infinity, NaN
-  if (s >= 0) return (unsigned long long)mant << s;
-  if (s < -24) return 0ull;                   // below one half
-  const int r = -s;                           // 1 .. 24
-  const uint32_t q = mant >> r, rem = mant & ((1u << r) - 1u), half = 1u << (r - 1);
-  return q + ((rem > half || (rem == half && (q & 1u))) ? 1u : 0u);
+  const int r = min(max(-s, 1), 31);
+  const uint32_t small = (mant + ((1u << (r - 1)) - 1u) + ((mant >> r) & 1u)) >> r;
+  const unsigned long long big = (unsigned long long)mant << min(max(s, 0), 40);
+  const unsigned long long wt = s >= 0 ? big : (unsigned long long)small;
+  return (e == 255 || s > 40) ? ~0ull : wt;      // at least 2^64, infinity, NaN
 }
 
 // Add a 64-bit weight to a histogram bin held as two 32-bit words (low,
