@@ -542,13 +542,19 @@ def measure_select(wl, hyper, K, V, Q, steps, warmup, ranks, M, LB, dev):
     time.sleep(0.3)
     torch.cuda.synchronize()
     ranks.barrier()
+    # the timed steps record no events between the kernels (so each kernel's
+    # launch overlaps the previous one's tail); the same number of steps
+    # with stage events follows for the per-stage times
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     t0.record(stream)
     for k in range(steps):
-        step(dbgs[k])
+        step()
     t1.record(stream)
     torch.cuda.synchronize()
     ranks.barrier()
+    for k in range(steps):
+        step(dbgs[k])
+    torch.cuda.synchronize()
     clk = clocks.stop()
     M.check(M.mmshift_poll_status(ws, stream), "timed status")
     ms = ranks.max(t0.elapsed_time(t1) / steps, dev)
@@ -764,13 +770,19 @@ def run_gpu(args, wl):
     time.sleep(0.3)
     torch.cuda.synchronize()
     ranks.barrier()
+    # the timed steps record no events between the kernels (so each kernel's
+    # launch overlaps the previous one's tail); the same number of steps
+    # with stage events follows for the per-stage times
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     t_start.record(stream)
     for k in range(args.steps):
-        step(dbgs[k], stat_ev[k])
+        step()
     t_end.record(stream)
     torch.cuda.synchronize()
     ranks.barrier()
+    for k in range(args.steps):
+        step(dbgs[k], stat_ev[k])
+    torch.cuda.synchronize()
     clk = clocks.stop()
     M.check(M.mmshift_poll_status(ws, stream), "timed status")
     ms = ranks.max(t_start.elapsed_time(t_end) / args.steps, dev)

@@ -367,7 +367,7 @@ static mmshift_status select_impl(const mmshift_shape* s, const void* K, const v
     bf.proxies_out = dbg->proxies;
     if (dbg->group_mass && P.G) bf.gmass = dbg->group_mass;
     if (dbg->anchor) bf.anchor = dbg->anchor;
-    if (dbg->scores) bf.scores = dbg->scores;
+    if (dbg->scores) { bf.scores = dbg->scores; bf.scores_out = 1; }
     bf.mass = dbg->mass;
   }
   const cudaStream_t cs = (cudaStream_t)stream;
@@ -582,7 +582,7 @@ mmshift_status mmshift_scores_topk(const mmshift_shape* s, const mmshift_params*
   if ((st = carve(P, workspace, workspace_bytes, &bf)) != MMSHIFT_OK) return st;
   if (P.G) bf.gmass = const_cast<float*>(group_mass);
   if (anchor) bf.anchor = const_cast<float*>(anchor);
-  if (scores) bf.scores = scores;
+  if (scores) { bf.scores = scores; bf.scores_out = 1; }
   const cudaStream_t cs = (cudaStream_t)stream;
   cudaError_t e = cudaSuccess;
   if (P.mode == MMSHIFT_SCORE_VOTE) e = launch_cover(P, bf, cs);

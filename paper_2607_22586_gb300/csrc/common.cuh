@@ -79,6 +79,7 @@ struct Buffers {
   float2* apart;      // [L][Hkv][total_splits][kMaxSplitAnchor] their (max, sum) per key split
   uint32_t* bits;     // [L][Hkv][G][total_words] coverage bitmaps
   float* scores;      // [L][Hkv][T]
+  int32_t scores_out; // the caller asked for the scores (else the top-k writes them only when it reads them back)
   float* mass;        // [L][Hkv][T] or null
   void* proxies_out;  // [L][B][Hq][Np][d] or null
   const void* proxies_in; // [L][B][Hq][Np][d] or null

@@ -70,6 +70,7 @@ extern "C" mmshift_status mmshift_scores_topk_noalloc(const mmshift_shape* s,
   bf.anchor = const_cast<float*>(anchor);
   bf.bits = static_cast<uint32_t*>(base);
   bf.scores = scores ? scores : reinterpret_cast<float*>(static_cast<char*>(base) + bits_bytes);
+  bf.scores_out = scores ? 1 : 0;
   const cudaStream_t cs = (cudaStream_t)stream;
   cudaError_t e = cudaSuccess;
   if (P.mode == MMSHIFT_SCORE_VOTE) e = launch_cover(P, bf, cs);

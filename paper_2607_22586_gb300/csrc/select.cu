@@ -1150,6 +1150,9 @@ __global__ void __launch_bounds__(NT, NT >= 1024 ? 1 : 2) topk_kernel(Problem P,
   const size_t hrow = ((size_t)l * P.Hkv + h) * P.total_T + R.tok_off;
   float* sc = bf.scores + hrow;
   const bool staged = n <= staged_cap;
+  // scores go to global memory when the selection reads them from there or
+  // the caller asked for them
+  const bool write_sc = !staged || bf.scores_out;
   // staged keys are counted by their 12-bit first digit as they are written
   // (select_kept_fine), the last key excepted
   if (staged) {
@@ -1166,8 +1169,9 @@ __global__ void __launch_bounds__(NT, NT >= 1024 ? 1 : 2) topk_kernel(Problem P,
     if (P.mode == MMSHIFT_SCORE_VOTE && P.G <= 8 && staged &&
         ((reinterpret_cast<uintptr_t>(an) | reinterpret_cast<uintptr_t>(sc)) & 15) == 0) {
       // four keys per lane: 16-byte loads of the anchors and stores of the
-      // scores and keys; a lane's keys 4j .. 4j+3 are bits (4j mod 32) .. +3
-      // of coverage word 4j / 32 (one word serves eight lanes)
+      // scores (if written) and keys; a lane's keys 4j .. 4j+3 are bits
+      // (4j mod 32) .. +3 of coverage word 4j / 32 (one word serves eight
+      // lanes)
       constexpr int UB4 = 4;
       const float4* an4 = reinterpret_cast<const float4*>(an);
       float4* sc4 = reinterpret_cast<float4*>(sc);
@@ -1202,7 +1206,7 @@ __global__ void __launch_bounds__(NT, NT >= 1024 ? 1 : 2) topk_kernel(Problem P,
             sv.y = __fadd_rn((float)((vt[u] >> 8) & 255u), __fmul_rn(P.lambda, a[u].y));
             sv.z = __fadd_rn((float)((vt[u] >> 16) & 255u), __fmul_rn(P.lambda, a[u].z));
             sv.w = __fadd_rn((float)(vt[u] >> 24), __fmul_rn(P.lambda, a[u].w));
-            sc4[j4] = sv;
+            if (write_sc) sc4[j4] = sv;
             const uint4 kq = make_uint4(nonneg_key(sv.x), nonneg_key(sv.y), nonneg_key(sv.z),
                                         nonneg_key(sv.w));
             ks4[j4] = kq;
@@ -1275,7 +1279,7 @@ __global__ void __launch_bounds__(NT, NT >= 1024 ? 1 : 2) topk_kernel(Problem P,
       for (int u = 0; u < UB; ++u) {
         const int i = base0 + u * NT + lane;
         if (i < n) {
-          sc[i] = sv[u];
+          if (write_sc) sc[i] = sv[u];
           if (staged) {
             const uint32_t kq = nonneg_key(sv[u]);
             keys_sm[i] = kq;
