@@ -116,6 +116,29 @@ def test_select_hyperparameters(kw):
     _check_all(wl, gpu, refs, h, what=str(kw))
 
 
+@pytest.mark.parametrize("kw", [dict(n_proxies=32, n_groups=2), dict(n_proxies=128, n_groups=32),
+                                dict(n_proxies=64, n_groups=4, tau=0.5)])
+def test_votes_exact_on_the_calls_own_masses(kw):
+    """The coverage vote of a full selection call (where the group totals
+    are known in advance, so its candidates come from the first pass) equals
+    the oracle's cover sets on the group masses the call itself computed,
+    key for key: the votes recovered from the scores (vote = S - lambda *
+    anchor, an integer) match O.votes(O.cover_sets(masses)) exactly."""
+    wl = QWEN1.replace(seq_lens=(6000, 900), n_visual=(5800, 850), budgets=(512, 100))
+    li = S.make_layer(wl, 1)
+    h = PT.hyper(**kw)
+    gpu = PT.gpu_select(wl, [li], h)
+    G, lam = h["n_groups"], np.float32(h["lam"])
+    for b, lo, hi, olo in _requests(wl):
+        for hh in range(wl.n_kv_heads):
+            gm = gpu["group_mass"][0][hh, :G, lo:hi].astype(np.float64)
+            v_own = O.votes(O.cover_sets(gm, h["tau"]))
+            an = gpu["anchor"][0][hh, lo:hi]
+            v_gpu = np.rint(gpu["scores"][0][hh, lo:hi].astype(np.float64) -
+                            (lam * an).astype(np.float32).astype(np.float64))
+            np.testing.assert_array_equal(v_gpu, v_own, err_msg=f"{kw} req {b} head {hh}")
+
+
 @pytest.mark.parametrize("lens", [(200, 333), (3000, 1333)])
 def test_multi_layer_call_matches_single_layer_calls(lens):
     """Bitwise equal whether the layers run in one call or one by one; the
