@@ -264,7 +264,8 @@ mmshift_status mmshift_proxy_mass(const mmshift_shape* s, const void* K, const v
  * first) holding at least tau of the group's mass --, votes, S_t = vote +
  * lambda * anchor (or sum_g mass in MASS mode), then the kept indices.
  * group_mass [L, Hkv, G, T], anchor [L, Hkv, T] (unused in MASS mode);
- * scores (nullable) [L, Hkv, T]; out_idx [L, R, Hkv]. */
+ * scores (nullable: S_t is written there when given) [L, Hkv, T];
+ * out_idx [L, R, Hkv]. */
 mmshift_status mmshift_scores_topk(const mmshift_shape* s, const mmshift_params* p,
                                    const float* group_mass, const float* anchor,
                                    float* scores, int32_t* out_idx,

@@ -56,7 +56,7 @@ struct Problem {
   // tensor-core path whose anchor rows would fill a 256-row softmax block of
   // their own (the group rows end on a block boundary): the softmax pass
   // leaves them out, the mass pass writes their scaled logits to alog and
-  // anchor_norm_kernel normalises them (set per call)
+  // anchor_part_kernel / anchor_final_kernel normalise them (set per call)
   int32_t anchor_split;
   // expected total of one group's masses over a request (its proxy rows:
   // each row's softmax sums to 1) when the coverage vote reads masses this
