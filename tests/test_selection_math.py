@@ -38,7 +38,8 @@ def weight_steps(bits: np.ndarray, shift: int) -> np.ndarray:
 
 
 def weight_reference(bits: np.ndarray, shift: int) -> np.ndarray:
-    x = bits.astype(np.uint32).view(np.float32).astype(np.float64)
+    with np.errstate(invalid="ignore"):   # NaN patterns (saturated below, as in the kernel)
+        x = bits.astype(np.uint32).view(np.float32).astype(np.float64)
     v = x * 2.0 ** shift
     out = np.empty(bits.shape, dtype=np.uint64)
     sat = ~np.isfinite(v) | (v >= 2.0 ** 64)
