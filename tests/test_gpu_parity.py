@@ -207,8 +207,9 @@ def test_end_to_end_sampled_bf16():
 # selection steps alone, on generated masses / scores (exact)
 # ---------------------------------------------------------------------------
 @pytest.mark.parametrize("tau", [0.95, 0.5, 1.0])
-def test_scores_topk_exact_on_generated_masses(tau):
-    wl = RAGGED.replace(seq_lens=(700, 2500, 40), n_visual=(600, 2400, 30), budgets=(100, 300, 8))
+def test_scores_topk_exact_on_generated_masses(tau, lens=(700, 2500, 40)):
+    # (only the lengths and budgets matter here: masses and anchors are generated)
+    wl = RAGGED.replace(seq_lens=lens, n_visual=tuple(0 for _ in lens), budgets=(100, 300, 8))
     h = PT.hyper(n_proxies=64, n_groups=8, tau=tau)
     T, hkv, G = wl.total_tokens, wl.n_kv_heads, h["n_groups"]
     gm = S.make_group_masses(hkv, G, T, 112.0, seed=5)
@@ -234,6 +235,13 @@ def test_scores_topk_exact_on_generated_masses(tau):
             np.testing.assert_array_equal(sc[hh, lo:hi], s_exp)
             np.testing.assert_array_equal(idx[olo:olo + keep, hh],
                                           O.select_topk(s_exp.astype(np.float64), wl.budgets[b]))
+
+
+@pytest.mark.parametrize("lens", [(701, 2498, 43), (3, 5, 1)])
+def test_scores_topk_exact_with_unaligned_requests(lens):
+    """Request offsets and lengths that are not multiples of four keys, so
+    the coverage vote's 16-byte passes start and end with scalar keys."""
+    test_scores_topk_exact_on_generated_masses(0.95, lens)
 
 
 @pytest.mark.parametrize("tau", [0.95, 0.5])
