@@ -416,6 +416,31 @@ def pin_cover_bruteforce(orc=O):
                     assert mass[g, t] > mass[g, u] or (mass[g, t] == mass[g, u] and t < u)
 
 
+def pin_cover_last_member_bound(orc=O):
+    """At realistic sizes: the tau-cover set is a prefix of the (mass desc, t
+    asc) order whose mass reaches tau * total while the same prefix without
+    its last member does not, and that last member's mass exceeds
+    (1 - tau) * total / n (the members before it hold less than tau * total,
+    the at most n - 1 keys after it at most its mass each)."""
+    rng = np.random.default_rng(23)
+    for n in (50, 700, 3000):
+        for tau in (0.5, 0.9, 0.95, 0.99):
+            mass = np.exp(rng.normal(0.0, 3.0, size=(3, n)))
+            mass[1, rng.random(n) < 0.5] = 0.0              # many zero keys
+            mass[2] = np.round(mass[2] * 4.0) / 4.0         # many ties
+            mass[2, 0] += 1.0
+            member = orc.cover_sets(mass, tau)
+            for g in range(3):
+                m, c = mass[g], member[g]
+                order = np.lexsort((np.arange(n), -m))
+                k = int(c.sum())
+                assert c[order[:k]].all() and not c[order[k:]].any()
+                total = m.sum()
+                assert m[order[:k]].sum() >= tau * total * (1 - 1e-12)
+                assert m[order[:k - 1]].sum() < tau * total
+                assert m[order[k - 1]] > (1.0 - tau) * total / n
+
+
 def pin_topk_bruteforce(orc=O):
     rng = np.random.default_rng(16)
     for trial in range(80):
@@ -542,7 +567,8 @@ ALL_PINS = [pin_philox_vs_numpy, pin_normals_distribution, pin_window_stats, pin
             pin_hidden_proxies, pin_attention_coverage, pin_head_budgets,
             pin_sampler_closed_form, pin_rope, pin_round_bf16, pin_mass_totals,
             pin_sigma_zero_single_query, pin_shift_and_permutation, pin_budget_ge_t,
-            pin_lastattn, pin_uniform_keys, pin_cover_bruteforce, pin_topk_bruteforce,
+            pin_lastattn, pin_uniform_keys, pin_cover_bruteforce, pin_cover_last_member_bound,
+            pin_topk_bruteforce,
             pin_mass_scores_bruteforce, pin_request_streams_and_slicing]
 
 
