@@ -58,7 +58,6 @@ struct SelShared {
   unsigned int digit;
   unsigned int prefix;
   unsigned int n_theta;
-  unsigned int max_key;
   unsigned int ncand;
   unsigned int rend;
   int aux;
@@ -338,16 +337,6 @@ __device__ void radix_passes(const Src& get, int n, int p0, int p1, uint32_t& pr
     prefix |= (S.digit & dmask) << sh;
     __syncthreads();
   }
-}
-
-template <bool WEIGHTED, int NTH, class Src>
-__device__ void radix_select(const Src& get, int n, unsigned long long target_w,
-                             unsigned target_n, int* shift, float tau, SelShared<NTH>& S,
-                             uint32_t* hist) {
-  uint32_t prefix = 0x80000000u;
-  radix_passes<WEIGHTED, NTH, Src>(get, n, 0, 4, prefix, target_w, target_n, shift, tau, S, hist);
-  if (threadIdx.x == 0) S.prefix = prefix;
-  __syncthreads();
 }
 
 // Copies the keys of get[0, n) whose bits at and above `hs` equal those of
